@@ -1,0 +1,298 @@
+"""CPU oracle for the Kashin-DCT decomposition and 2-bit coding (TEST INFRASTRUCTURE).
+
+This module is the slow, plain, obviously-correct reference that the CUDA path is
+checked against.  It is test infrastructure: only ``tests/``,
+``__graft_entry__.smoke()`` and ``bench.py``'s CPU-baseline leg may import it, and
+the library never calls it.  It shares no code with the CUDA path: no fast
+transform, no factorisation, no tables.
+
+Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
+
+* ``dct2_matrix``          -- orthonormal DCT-II (Sec. 3.1, footnote on ``norm='ortho'``;
+                              App. C footnote).  Row 0 carries the extra ``1/sqrt 2``
+                              that makes the matrix orthogonal (reading c-1).
+* ``sign_mask``            -- the per-matrix sign set ``epsilon`` (Sec. 3.1 ``T_E``;
+                              App. C "generated once from a fixed seed").  The paper
+                              does not name its generator; this build reads it as
+                              SplitMix64 (Steele, Lea & Flood, OOPSLA 2014): bit 63 of
+                              the mix of ``seed + (j + 1) * gamma`` set means -1.
+* ``apply_p``              -- ``P z = IDCT(eps * DCT(z))`` with the dense matrix (Alg. 1).
+* ``decompose``            -- Algorithm 1 (Greedy Algorithm with Alternating Updates)
+                              written out step by step, with ``sign(0) = 0`` and the
+                              step divisor ``N`` as printed.  Optional tie-follow.
+* ``centres`` / ``codes``  -- the closed-form centres +-c1 +-c2 (Sec. 2.1) and the
+                              nearest-centre 2-bit code (Sec. 2.1, App. C).
+* ``reconstruct``          -- dequantised ``W_hat = U_q + P V_q`` (App. C, Eq. 11).
+
+Parity pins (tests/test_oracle_pins.py) tie each function to something the paper
+or mathematics fixes; the ``l_inf`` bound constant of Theorem 2 contains the
+unknown ``c_3`` and is *parity unpinned* as a number (only the coefficient-sum
+form of the bound is checked).
+"""
+
+from __future__ import annotations
+
+import dataclasses
+from typing import Optional
+
+import numpy as np
+
+# ---------------------------------------------------------------------------
+# Orthonormal DCT-II and the sign-randomised operator P (Sec. 3.1, App. C)
+# ---------------------------------------------------------------------------
+
+
+def dct2_matrix(N: int) -> np.ndarray:
+    """Orthonormal DCT-II matrix ``C[j, n] = s_j sqrt(2/N) cos(pi (2n+1) j / (2N))``.
+
+    ``s_0 = 1/sqrt(2)``, ``s_j = 1`` otherwise (Sec. 3.1 basis ``phi_j`` with the
+    ``norm='ortho'`` convention of the footnote), so ``C^T = C^{-1}``.
+    """
+    n = np.arange(N, dtype=np.float64)[None, :]
+    j = np.arange(N, dtype=np.float64)[:, None]
+    C = np.sqrt(2.0 / N) * np.cos(np.pi * (2.0 * n + 1.0) * j / (2.0 * N))
+    C[0, :] *= 1.0 / np.sqrt(2.0)
+    return C
+
+
+_MASK64 = (1 << 64) - 1
+_GAMMA = 0x9E3779B97F4A7C15
+
+
+def splitmix64(state: int) -> int:
+    """SplitMix64 output function applied to a 64-bit state (Steele, Lea & Flood 2014)."""
+    z = state & _MASK64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _MASK64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _MASK64
+    return z ^ (z >> 31)
+
+
+def sign_mask(seed: int, N: int) -> np.ndarray:
+    """``epsilon_j`` for DCT coefficient ``j`` (0-based): +1, or -1 where bit 63 of
+    ``splitmix64(seed + (j + 1) * gamma)`` is set.  One mask per matrix, shared by
+    all its columns (App. C)."""
+    out = np.empty(N, dtype=np.float64)
+    s = int(seed) & _MASK64
+    for j in range(N):
+        z = splitmix64((s + (j + 1) * _GAMMA) & _MASK64)
+        out[j] = -1.0 if (z >> 63) else 1.0
+    return out
+
+
+def p_matrix(N: int, eps: np.ndarray) -> np.ndarray:
+    """Dense ``P = C^T diag(eps) C`` (the operator U_{E,Phi} of Sec. 3.1)."""
+    C = dct2_matrix(N)
+    return C.T @ (eps[:, None] * C)
+
+
+class POperator:
+    """``P z = IDCT(eps * DCT(z))`` applied with the explicit DCT matrix (Alg. 1)."""
+
+    def __init__(self, N: int, eps: np.ndarray):
+        self.N = N
+        self.eps = np.asarray(eps, dtype=np.float64)
+        self.C = dct2_matrix(N)
+
+    def __call__(self, z: np.ndarray) -> np.ndarray:
+        z = np.asarray(z, dtype=np.float64)
+        a = self.C @ z                       # DCT
+        if a.ndim == 1:
+            a = self.eps * a                 # T_eps
+        else:
+            a = self.eps[:, None] * a
+        return self.C.T @ a                  # IDCT = DCT^T
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 1: Greedy Algorithm with Alternating Updates
+# ---------------------------------------------------------------------------
+
+
+@dataclasses.dataclass
+class Decomposition:
+    u: np.ndarray          # (N, M)
+    vhat: np.ndarray       # (N, M), P-domain factor; v = P vhat
+    r: np.ndarray          # (N, M) residual r_k
+    coeffs: np.ndarray     # (4, M): c1, c2 (block 0, steps 1-2), d1, d2 (block 0, steps 3-4)
+    lambdas: np.ndarray    # (4k, M): coefficient of every atomic step
+    step_norms: np.ndarray  # (4k + 1, M): ||rho||_2 entering each step, then final
+    ties: int = 0          # decisions taken from the followed trace (|arg| <= tau)
+    tie_flips: int = 0     # ... of which the followed sign differs from the oracle's own
+    hard_mismatches: int = 0  # |arg| > tau but the followed sign differs (parity failure)
+
+
+def _sign(a: np.ndarray) -> np.ndarray:
+    """``sign`` with ``sign(0) = 0`` (reading c-2)."""
+    return np.sign(a)
+
+
+def decompose(x: np.ndarray, eps: np.ndarray, iters: int, follow: Optional[np.ndarray] = None,
+              tau_abs: Optional[np.ndarray] = None, P: Optional[POperator] = None) -> Decomposition:
+    """Run Algorithm 1 on every column of ``x`` (shape ``(N, M)``), float64.
+
+    Per block t (k blocks): two greedy steps on the cube vertices Q_N update u,
+    then two steps on P Q_N update vhat, exactly as Alg. 1 prints them::
+
+        Delta_u    = sign(rho) * ||rho||_1 / N ;  u += Delta_u ;     rho -= Delta_u
+        Delta_vhat = sign(P rho) * ||P rho||_1 / N ; vhat += Delta_vhat ; rho -= P Delta_vhat
+
+    Tie-follow (test protocol for the discontinuous ``sign``): if ``follow`` is
+    given (int8, shape ``(4k, N, M)``: the sign the device took at every atomic
+    step, in natural element order), then wherever the oracle's own argument has
+    ``|arg| <= tau_abs[col]`` the followed sign is used instead; a disagreement
+    where ``|arg| > tau_abs`` is counted in ``hard_mismatches``.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    if x.ndim == 1:
+        x = x[:, None]
+    N, M = x.shape
+    if P is None:
+        P = POperator(N, eps)
+    u = np.zeros_like(x)
+    vhat = np.zeros_like(x)
+    r = x.copy()
+    coeffs = np.zeros((4, M))
+    lambdas = np.zeros((4 * iters, M))
+    norms = np.zeros((4 * iters + 1, M))
+    stats = {"ties": 0, "flips": 0, "hard": 0}
+
+    def choose_sign(arg: np.ndarray, step: int) -> np.ndarray:
+        own = _sign(arg)
+        if follow is None:
+            return own
+        dev = follow[step].astype(np.float64)
+        near = np.abs(arg) <= tau_abs[None, :]
+        stats["ties"] += int(near.sum())
+        stats["flips"] += int((near & (dev != own)).sum())
+        stats["hard"] += int((~near & (dev != own)).sum())
+        return np.where(near, dev, own)
+
+    step = 0
+    for t in range(iters):
+        rho = r.copy()
+        for j in (1, 2):                     # two greedy steps from Q_N
+            norms[step] = np.linalg.norm(rho, axis=0)
+            lam = np.abs(rho).sum(axis=0) / N
+            du = choose_sign(rho, step) * lam[None, :]
+            u = u + du
+            rho = rho - du
+            lambdas[step] = lam
+            if t == 0:
+                coeffs[j - 1] = lam
+            step += 1
+        for j in (3, 4):                     # two greedy steps from P Q_N
+            norms[step] = np.linalg.norm(rho, axis=0)
+            y = P(rho)
+            lam = np.abs(y).sum(axis=0) / N
+            dv = choose_sign(y, step) * lam[None, :]
+            vhat = vhat + dv
+            rho = rho - P(dv)
+            lambdas[step] = lam
+            if t == 0:
+                coeffs[j - 1] = lam
+            step += 1
+        r = rho
+    norms[step] = np.linalg.norm(r, axis=0)
+    return Decomposition(u=u, vhat=vhat, r=r, coeffs=coeffs, lambdas=lambdas, step_norms=norms,
+                         ties=stats["ties"], tie_flips=stats["flips"], hard_mismatches=stats["hard"])
+
+
+# ---------------------------------------------------------------------------
+# Closed-form centres and 2-bit codes (Sec. 2.1, App. C)
+# ---------------------------------------------------------------------------
+
+
+def centres(a1: np.ndarray, a2: np.ndarray) -> np.ndarray:
+    """The four peaks +-a1 +-a2 of a factor after its two block-0 updates, ascending.
+
+    Returns shape ``(M, 4)``: ``[-(a1+a2), -|a1-a2|, |a1-a2|, a1+a2]``."""
+    a1 = np.asarray(a1, dtype=np.float64)
+    a2 = np.asarray(a2, dtype=np.float64)
+    outer = a1 + a2
+    inner = np.abs(a1 - a2)
+    return np.stack([-outer, -inner, inner, outer], axis=-1)
+
+
+def codes(values: np.ndarray, cent: np.ndarray) -> np.ndarray:
+    """Index of the nearest centre for every entry (ties to the lower index).
+
+    ``values`` has shape ``(N, M)``, ``cent`` shape ``(M, 4)`` ascending.  The
+    decision is taken in float32 (the precision the device decides in): both
+    the values and the centre midpoints are rounded to float32 first.  Each
+    boundary is the midpoint of two adjacent centres.
+    """
+    v32 = np.asarray(values, dtype=np.float32)
+    c32 = np.asarray(cent, dtype=np.float64)
+    b = np.stack([(c32[:, 0] + c32[:, 1]) / 2, (c32[:, 1] + c32[:, 2]) / 2,
+                  (c32[:, 2] + c32[:, 3]) / 2], axis=-1).astype(np.float32)  # (M, 3)
+    out = np.zeros(v32.shape, dtype=np.int64)
+    for i in range(3):
+        out += (v32 > b[None, :, i]).astype(np.int64)
+    return out
+
+
+def boundary_distance(values: np.ndarray, cent: np.ndarray) -> np.ndarray:
+    """Distance of every entry to its nearest decision boundary (float64)."""
+    c = np.asarray(cent, dtype=np.float64)
+    b = np.stack([(c[:, 0] + c[:, 1]) / 2, (c[:, 1] + c[:, 2]) / 2, (c[:, 2] + c[:, 3]) / 2], axis=-1)
+    v = np.asarray(values, dtype=np.float64)
+    return np.min(np.abs(v[:, :, None] - b[None, :, :]), axis=-1)
+
+
+def pack_codes(code: np.ndarray) -> np.ndarray:
+    """Pack 2-bit codes of shape ``(N, M)`` into ``(M, ceil(N/16))`` uint32 words:
+    entry i of a column sits at bits ``2 (i mod 16)`` of word ``i // 16``."""
+    N, M = code.shape
+    W = (N + 15) // 16
+    out = np.zeros((M, W), dtype=np.uint64)
+    for i in range(N):
+        out[:, i // 16] |= (code[i, :].astype(np.uint64) & 3) << np.uint64(2 * (i % 16))
+    return out.astype(np.uint32)
+
+
+def unpack_codes(words: np.ndarray, N: int) -> np.ndarray:
+    """Inverse of :func:`pack_codes`: returns ``(N, M)`` int64 codes."""
+    words = np.asarray(words, dtype=np.uint64)
+    M = words.shape[0]
+    out = np.zeros((N, M), dtype=np.int64)
+    for i in range(N):
+        out[i, :] = (words[:, i // 16] >> np.uint64(2 * (i % 16))) & np.uint64(3)
+    return out
+
+
+def dequantise(code: np.ndarray, cent: np.ndarray) -> np.ndarray:
+    """``c[code]`` per column: ``(N, M)`` codes with ``(M, 4)`` centres."""
+    M = cent.shape[0]
+    return np.asarray(cent, dtype=np.float64)[np.arange(M)[None, :], code]
+
+
+def reconstruct(code_u: np.ndarray, code_v: np.ndarray, cent_u: np.ndarray, cent_v: np.ndarray,
+                eps: np.ndarray) -> np.ndarray:
+    """Dequantised weight ``W_hat = U_q + P V_q`` (App. C: dense re-materialisation)."""
+    uq = dequantise(code_u, cent_u)
+    vq = dequantise(code_v, cent_v)
+    P = POperator(uq.shape[0], eps)
+    return uq + P(vq)
+
+
+@dataclasses.dataclass
+class Quantised:
+    dec: Decomposition
+    centres_u: np.ndarray   # (M, 4)
+    centres_v: np.ndarray   # (M, 4)
+    codes_u: np.ndarray     # (N, M)
+    codes_v: np.ndarray     # (N, M)
+
+
+def quantise(x: np.ndarray, seed: int, iters: int, follow: Optional[np.ndarray] = None,
+             tau_abs: Optional[np.ndarray] = None) -> Quantised:
+    """Decompose every column (Alg. 1), then code each factor with its closed-form
+    centres (Sec. 2.1): u with (c1, c2), vhat with (d1, d2), zero refinement
+    iterations (reading c-6)."""
+    x = np.asarray(x, dtype=np.float64)
+    eps = sign_mask(seed, x.shape[0])
+    dec = decompose(x, eps, iters, follow=follow, tau_abs=tau_abs)
+    cu = centres(dec.coeffs[0], dec.coeffs[1])
+    cv = centres(dec.coeffs[2], dec.coeffs[3])
+    return Quantised(dec=dec, centres_u=cu, centres_v=cv, codes_u=codes(dec.u, cu),
+                     codes_v=codes(dec.vhat, cv))
