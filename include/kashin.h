@@ -1,0 +1,134 @@
+/*
+ * libkashin -- C ABI of the GB300 (sm_103a) Kashin-DCT decomposition and 2-bit coder.
+ *
+ * The method (arxiv 2609.11687, "Structured Transforms for Low-Overhead
+ * Quantization of Language Models"):
+ *   - every weight vector x of length n (a column of the paper's n x m matrix W,
+ *     App. C) is decomposed by Algorithm 1 (Greedy Algorithm with Alternating
+ *     Updates) into  x = u + P vhat + r,  P = IDCT o T_eps o DCT  (Sec. 3.1), with
+ *     the orthonormal DCT-II and one sign set eps in {+-1}^n per matrix drawn from
+ *     a seed (App. C);
+ *   - each factor is coded to 2 bits with the closed-form centres +-c1 +-c2
+ *     (u, from the two u-steps of block 0) and +-d1 +-d2 (vhat, from the two
+ *     vhat-steps of block 0), nearest centre, ties to the lower code (Sec. 2.1);
+ *   - the dequantised weight is  W_hat = U_q + P V_q  (App. C, dense
+ *     re-materialisation at load time).
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  n       vector length (the paper's N: rows of W, input features).
+ *  m       number of vectors (the paper's M: columns of W, output channels).
+ *  layout  KD_VEC_ROWS:    vector j is w[j*ld + i], i < n  (row-major m x ld, ld >= n;
+ *                          the nn.Linear weight layout [out, in]).
+ *          KD_VEC_COLUMNS: vector j is w[i*ld + j], i < n  (row-major n x ld, ld >= m;
+ *                          the paper's N x M matrix).
+ *  sign seed   eps_j = +1, or -1 where bit 63 of SplitMix64(seed + (j+1)*0x9E3779B97F4A7C15)
+ *              is set (SplitMix64: Steele, Lea & Flood, OOPSLA 2014).  The paper
+ *              does not name its generator; this is the library's fixed choice.
+ *  Pointers    every array argument is DEVICE memory owned by the caller unless
+ *              it is named *_host.  The library allocates nothing per call.
+ *  stream      a cudaStream_t passed as void* (NULL = legacy default stream).
+ *              Calls validate their arguments synchronously, then only enqueue
+ *              work on the stream and return.
+ *  Errors      argument / size / plan problems are returned synchronously and
+ *              nothing is enqueued; a failed launch returns KD_ERR_CUDA; a
+ *              non-finite input value is detected on the device and reported
+ *              by kd_read_status().  No call traps or aborts.
+ *  Supported n: n even, 16 <= n <= 16384, with a compiled plan (kd_supported());
+ *              at least 256, 512, 768, 1024, 1536, 2048, 3072, 4096, 8192,
+ *              11008, 14336, 16384.
+ */
+#ifndef KASHIN_H
+#define KASHIN_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  KD_OK = 0,
+  KD_ERR_INVALID_ARG = 1,   /* null required pointer, bad size, bad enum, ld too small */
+  KD_ERR_UNSUPPORTED_N = 2, /* no compiled plan for this vector length */
+  KD_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed */
+  KD_ERR_NONFINITE = 4,     /* a decomposed vector held NaN or Inf (device-detected) */
+  KD_ERR_WORKSPACE = 5      /* workspace pointer null or smaller than kd_workspace_size() */
+} kd_status;
+
+typedef enum { KD_F32 = 0, KD_F16 = 1, KD_BF16 = 2 } kd_dtype;
+
+typedef enum { KD_VEC_ROWS = 0, KD_VEC_COLUMNS = 1 } kd_layout;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char* kd_status_string(kd_status s);
+
+/* Library version string. */
+const char* kd_version(void);
+
+/* KD_OK if vector length n has a compiled plan, else KD_ERR_UNSUPPORTED_N. */
+kd_status kd_supported(int64_t n);
+
+/* Bytes of device workspace kd_decompose / kd_apply_p / kd_reconstruct need for
+ * vector length n on the current device (0 if n is unsupported).  The workspace
+ * holds the per-call sign mask, the transform twiddles and a device status word;
+ * it must stay allocated until the enqueued work completes and must not be
+ * shared by calls in flight on different streams. */
+size_t kd_workspace_size(int64_t n);
+
+/* The sign set eps of Sec. 3.1 / App. C for a seed, on the host:
+ * eps_host[j] = +1 or -1, j < n.  Pure host computation, no CUDA call. */
+kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host);
+
+/* Algorithm 1 on every vector of w, then the closed-form 2-bit coding of both
+ * factors (Sec. 3.2 Algorithm 1; Sec. 2.1; App. C storage format).
+ *
+ *  w          input, dtype elements, `layout` with leading dimension ld.
+ *  iters      k >= 0 blocks of four atomic greedy steps (two on Q_N -> u, two on
+ *             P Q_N -> vhat).  k = 0 gives zero factors, zero centres, codes 0.
+ *  codes_u,   required, uint32[m][ceil(n/16)]: 2-bit code of u_i (resp. vhat_i) at
+ *  codes_v    bits 2*(i%16) of word i/16 of vector j's row; code c indexes the
+ *             ascending centre table.
+ *  centres_u, required, float[m][4] ascending: -(a1+a2), -|a1-a2|, |a1-a2|, a1+a2
+ *  centres_v  with (a1, a2) = (c1, c2) for u and (d1, d2) for vhat.
+ *  coeffs     optional, float[m][4]: c1, c2, d1, d2 (block-0 step coefficients).
+ *  u, vhat,   optional, float[m][n] (vector-major, contiguous): the factors u_k,
+ *  resid      vhat_k and the residual r_k of Algorithm 1, x = u + P vhat + r.
+ *  trace      optional, int8[m][4*iters][n]: sign(.) in {-1, 0, +1} that every
+ *             atomic step applied to element i (natural order).  Test/debug
+ *             output; enabling it does not change any other output bit.
+ *  workspace  device scratch of ws_bytes >= kd_workspace_size(n).
+ *
+ * Vectors are processed two at a time (2j, 2j+1); each vector's results depend
+ * only on its own data and its pair partner's (through rounding only). */
+kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
+                       int64_t ld, uint64_t sign_seed, int iters,
+                       uint32_t* codes_u, uint32_t* codes_v, float* centres_u, float* centres_v,
+                       float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
+                       void* workspace, size_t ws_bytes, void* stream);
+
+/* y_j = P x_j for m vectors of length n, fp32, vector-major [m][n] contiguous
+ * (Sec. 3.1: P z = IDCT(eps * DCT(z)); App. C uses the same operator on the rows
+ * of the activations, XP).  x and y may alias. */
+kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t sign_seed,
+                     void* workspace, size_t ws_bytes, void* stream);
+
+/* Dense re-materialisation W_hat = U_q + P V_q (App. C): vector j of w_hat is
+ * centres_u[j][code_u] + P(centres_v[j][code_v]).  Inputs as produced by
+ * kd_decompose; output dtype out_dtype in `layout` with leading dimension ld. */
+kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v,
+                         const float* centres_u, const float* centres_v, int64_t n, int64_t m,
+                         uint64_t sign_seed, kd_dtype out_dtype, kd_layout layout, void* w_hat,
+                         int64_t ld, void* workspace, size_t ws_bytes, void* stream);
+
+/* Synchronises `stream` and returns KD_ERR_NONFINITE if any vector decomposed
+ * by the last kd_decompose on this workspace held a NaN or Inf, KD_OK otherwise
+ * (KD_ERR_CUDA if the synchronisation fails). */
+kd_status kd_read_status(const void* workspace, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KASHIN_H */

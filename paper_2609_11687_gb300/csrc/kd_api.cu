@@ -1,0 +1,290 @@
+// C ABI of libkashin (declared in include/kashin.h): argument validation, the
+// per-call workspace layout, table set-up and kernel dispatch by vector length.
+#include <cstring>
+
+#include "kashin.h"
+#include "kd_kernels.cuh"
+#include "kd_ops.h"
+
+namespace kd {
+#define KD_PLAN(n) const PlanOps* plan_ops_##n();
+KD_PLAN(16) KD_PLAN(32) KD_PLAN(64) KD_PLAN(128) KD_PLAN(256) KD_PLAN(512) KD_PLAN(768)
+KD_PLAN(1024) KD_PLAN(1536) KD_PLAN(2048) KD_PLAN(3072) KD_PLAN(4096) KD_PLAN(8192)
+KD_PLAN(11008) KD_PLAN(14336) KD_PLAN(16384)
+#undef KD_PLAN
+
+const PlanOps* plan_ops(int64_t n) {
+  switch (n) {
+    case 16: return plan_ops_16();
+    case 32: return plan_ops_32();
+    case 64: return plan_ops_64();
+    case 128: return plan_ops_128();
+    case 256: return plan_ops_256();
+    case 512: return plan_ops_512();
+    case 768: return plan_ops_768();
+    case 1024: return plan_ops_1024();
+    case 1536: return plan_ops_1536();
+    case 2048: return plan_ops_2048();
+    case 3072: return plan_ops_3072();
+    case 4096: return plan_ops_4096();
+    case 8192: return plan_ops_8192();
+    case 11008: return plan_ops_11008();
+    case 14336: return plan_ops_14336();
+    case 16384: return plan_ops_16384();
+    default: return nullptr;
+  }
+}
+
+namespace {
+
+// ---------------------------------------------------------------------------
+// Per-call tables: twiddles W_{2N}^j (double-precision sincospi, rounded) and the
+// sign mask bits (SplitMix64 of seed + (j+1)*gamma, bit 63 set -> eps_j = -1).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__global__ void setup_tables_kernel(float2* tw, uint32_t* eps, uint32_t* status, int n, uint64_t seed) {
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int stride = gridDim.x * blockDim.x;
+  if (tid == 0) *status = 0u;
+  for (int j = tid; j < 2 * n; j += stride) {
+    double s, c;
+    sincospi((double)j / (double)n, &s, &c);
+    tw[j] = make_float2((float)c, (float)(-s));
+  }
+  const int words = (n + 31) / 32;
+  for (int wd = tid; wd < words; wd += stride) {
+    uint32_t bits = 0;
+    for (int b = 0; b < 32; ++b) {
+      const int j = wd * 32 + b;
+      if (j >= n) break;
+      const uint64_t z = splitmix64_mix(seed + (uint64_t)(j + 1) * 0x9E3779B97F4A7C15ull);
+      bits |= (uint32_t)(z >> 63) << b;
+    }
+    eps[wd] = bits;
+  }
+}
+
+
+constexpr size_t kAlign = 256;
+inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
+
+// Workspace layout: [status word | pad][twiddles 2n float2][sign bits][u slots]
+struct WsLayout {
+  size_t status, tw, eps, uslots, total;
+};
+
+int sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return sms;
+}
+
+// Most CTAs a decompose launch of this plan ever uses on the current device.
+int max_decompose_ctas(const PlanOps* ops) {
+  const int per = ops->ctas_per_sm(0);
+  const int sms = sm_count();
+  if (per <= 0 || sms <= 0) return 0;
+  return per * sms;
+}
+
+bool layout_of(const PlanOps* ops, WsLayout* L) {
+  const size_t n = (size_t)ops->n;
+  L->status = 0;
+  L->tw = kAlign;
+  L->eps = L->tw + align_up(2 * n * sizeof(float2));
+  L->uslots = L->eps + align_up(((n + 31) / 32) * sizeof(uint32_t));
+  size_t us = 0;
+  if (ops->u_in_gmem) {
+    const int ctas = max_decompose_ctas(ops);
+    if (ctas <= 0) return false;
+    us = align_up((size_t)ctas * ops->q * n * sizeof(float2));
+  }
+  L->total = L->uslots + us;
+  return true;
+}
+
+kd_status setup(const PlanOps* ops, const WsLayout& L, void* ws, uint64_t seed, cudaStream_t s) {
+  char* b = static_cast<char*>(ws);
+  const int n = ops->n;
+  const int threads = 256;
+  const int blocks = (2 * n + threads - 1) / threads;
+  setup_tables_kernel<<<blocks, threads, 0, s>>>(reinterpret_cast<float2*>(b + L.tw),
+                                                 reinterpret_cast<uint32_t*>(b + L.eps),
+                                                 reinterpret_cast<uint32_t*>(b + L.status), n, seed);
+  return cudaGetLastError() == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+int grid_for(int64_t npairs, int q, int ctas_max) {
+  const int64_t want = (npairs + q - 1) / q;
+  return (int)(want < ctas_max ? want : ctas_max);
+}
+
+bool valid_dtype(int d) { return d == KD_F32 || d == KD_F16 || d == KD_BF16; }
+bool valid_layout(int l) { return l == KD_VEC_ROWS || l == KD_VEC_COLUMNS; }
+
+}  // namespace
+}  // namespace kd
+
+using namespace kd;
+
+extern "C" {
+
+const char* kd_status_string(kd_status s) {
+  switch (s) {
+    case KD_OK: return "KD_OK";
+    case KD_ERR_INVALID_ARG: return "KD_ERR_INVALID_ARG";
+    case KD_ERR_UNSUPPORTED_N: return "KD_ERR_UNSUPPORTED_N";
+    case KD_ERR_CUDA: return "KD_ERR_CUDA";
+    case KD_ERR_NONFINITE: return "KD_ERR_NONFINITE";
+    case KD_ERR_WORKSPACE: return "KD_ERR_WORKSPACE";
+    default: return "KD_ERR_UNKNOWN";
+  }
+}
+
+const char* kd_version(void) { return "libkashin 0.1.0 (sm_103a)"; }
+
+kd_status kd_supported(int64_t n) { return plan_ops(n) ? KD_OK : KD_ERR_UNSUPPORTED_N; }
+
+size_t kd_workspace_size(int64_t n) {
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return 0;
+  WsLayout L;
+  if (!layout_of(ops, &L)) return 0;
+  return L.total;
+}
+
+kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host) {
+  if (n <= 0 || !eps_host) return KD_ERR_INVALID_ARG;
+  for (int64_t j = 0; j < n; ++j) {
+    uint64_t z = sign_seed + (uint64_t)(j + 1) * 0x9E3779B97F4A7C15ull;
+    z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+    z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+    z = z ^ (z >> 31);
+    eps_host[j] = (z >> 63) ? (int8_t)-1 : (int8_t)1;
+  }
+  return KD_OK;
+}
+
+kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m, int64_t ld,
+                       uint64_t sign_seed, int iters, uint32_t* codes_u, uint32_t* codes_v,
+                       float* centres_u, float* centres_v, float* coeffs, float* u, float* vhat,
+                       float* resid, int8_t* trace, void* workspace, size_t ws_bytes, void* stream) {
+  if (n <= 0 || m < 0 || iters < 0 || !valid_dtype(dtype) || !valid_layout(layout)) return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
+  if (m > 0 && (!w || !codes_u || !codes_v || !centres_u || !centres_v)) return KD_ERR_INVALID_ARG;
+  WsLayout L;
+  if (!layout_of(ops, &L)) return KD_ERR_CUDA;
+  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  kd_status st = setup(ops, L, workspace, sign_seed, s);
+  if (st != KD_OK || m == 0) return st;
+  char* b = static_cast<char*>(workspace);
+  DecParams p;
+  p.w = w;
+  p.dtype = (int)dtype;
+  p.layout = (int)layout;
+  p.n = n;
+  p.m = m;
+  p.ld = ld;
+  p.iters = iters;
+  p.codes_u = codes_u;
+  p.codes_v = codes_v;
+  p.centres_u = centres_u;
+  p.centres_v = centres_v;
+  p.coeffs = coeffs;
+  p.u = u;
+  p.vhat = vhat;
+  p.resid = resid;
+  p.trace = trace;
+  p.tw = reinterpret_cast<const float2*>(b + L.tw);
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.status = reinterpret_cast<uint32_t*>(b + L.status);
+  p.uslots = ops->u_in_gmem ? reinterpret_cast<float2*>(b + L.uslots) : nullptr;
+  p.npairs = (m + 1) / 2;
+  const int ctas = max_decompose_ctas(ops);
+  if (ctas <= 0) return KD_ERR_CUDA;
+  const int grid = grid_for(p.npairs, ops->q, ctas);
+  return ops->decompose(p, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t sign_seed, void* workspace,
+                     size_t ws_bytes, void* stream) {
+  if (n <= 0 || m < 0) return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  if (m > 0 && (!x || !y)) return KD_ERR_INVALID_ARG;
+  WsLayout L;
+  if (!layout_of(ops, &L)) return KD_ERR_CUDA;
+  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  kd_status st = setup(ops, L, workspace, sign_seed, s);
+  if (st != KD_OK || m == 0) return st;
+  char* b = static_cast<char*>(workspace);
+  ApplyParams p;
+  p.x = x;
+  p.y = y;
+  p.m = m;
+  p.tw = reinterpret_cast<const float2*>(b + L.tw);
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.npairs = (m + 1) / 2;
+  const int per = ops->ctas_per_sm(1);
+  const int sms = sm_count();
+  if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
+  const int grid = grid_for(p.npairs, ops->q, per * sms);
+  return ops->apply(p, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
+                         const float* centres_v, int64_t n, int64_t m, uint64_t sign_seed, kd_dtype out_dtype,
+                         kd_layout layout, void* w_hat, int64_t ld, void* workspace, size_t ws_bytes,
+                         void* stream) {
+  if (n <= 0 || m < 0 || !valid_dtype(out_dtype) || !valid_layout(layout)) return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
+  if (m > 0 && (!codes_u || !codes_v || !centres_u || !centres_v || !w_hat)) return KD_ERR_INVALID_ARG;
+  WsLayout L;
+  if (!layout_of(ops, &L)) return KD_ERR_CUDA;
+  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  kd_status st = setup(ops, L, workspace, sign_seed, s);
+  if (st != KD_OK || m == 0) return st;
+  char* b = static_cast<char*>(workspace);
+  RecParams p;
+  p.dtype = (int)out_dtype;
+  p.layout = (int)layout;
+  p.codes_u = codes_u;
+  p.codes_v = codes_v;
+  p.centres_u = centres_u;
+  p.centres_v = centres_v;
+  p.m = m;
+  p.ld = ld;
+  p.out = w_hat;
+  p.tw = reinterpret_cast<const float2*>(b + L.tw);
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.npairs = (m + 1) / 2;
+  const int per = ops->ctas_per_sm(2);
+  const int sms = sm_count();
+  if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
+  const int grid = grid_for(p.npairs, ops->q, per * sms);
+  return ops->reconstruct(p, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+kd_status kd_read_status(const void* workspace, void* stream) {
+  if (!workspace) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  uint32_t word = 0;
+  if (cudaMemcpyAsync(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess) return KD_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return KD_ERR_CUDA;
+  return word ? KD_ERR_NONFINITE : KD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,677 @@
+// Kashin-DCT decomposition kernels (sm_103a).
+//
+// One team of T threads owns a PAIR of vectors (2j, 2j+1) for the whole of
+// Algorithm 1: the two real vectors are the real and imaginary parts of one
+// complex vector held on-chip, so one complex FFT of length N transforms both.
+//
+// Transform (Sec. 3.1, Alg. 1: P z = IDCT(eps * DCT(z))).  With the vector held
+// in Makhoul's even/odd order v[p] = x[2p], v[N-1-p] = x[2p+1] (J. Makhoul, IEEE
+// TASSP 1980) the orthonormal DCT-II is Re(exp(-i pi k / 2N) DFT(v)_k) up to a
+// per-k scale that cancels in IDCT o T_eps o DCT, and P becomes
+//     P' z = IDFT( M( DFT(z) ) ),
+//     M: Z'_k = e+_k Z_k + e-_k exp(i pi k/N) Z_{N-k},  e+-_k = (eps_k +- eps_{N-k})/2,
+//        Z'_0 = eps_0 Z_0,  Z'_{N/2} = eps_{N/2} Z_{N/2},
+// which is complex-linear, so it acts on both packed vectors at once.
+//
+// The greedy steps (sign, l1 norm, update) are permutation-invariant, so the
+// vectors stay in Makhoul order in the "spatial" domain for all k blocks: the
+// forward FFT runs decimation-in-frequency (natural in, digit-reversed out), M
+// pairs digit-reversed slots, and the inverse runs the mirror passes back to
+// natural order -- no reordering pass exists anywhere.
+//
+// Data layout per team: the spatial vector lives in registers, E = R0 complex
+// values per thread at positions t + j*T (which is exactly the first radix
+// pass's group), and a padded shared-memory buffer of N float2 carries the
+// exchanges between radix passes.  The factor u lives in registers (small E) or
+// in a per-team slot of the workspace (large N).  vhat is not stored during the
+// loop: after the last block it is recovered as P(x - u - r) (P^2 = I).
+#pragma once
+
+#include <cstdint>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+
+#include "kd_math.cuh"
+
+namespace kd {
+
+enum { UREG = 0, UGMEM = 1 };
+enum { DT_F32 = 0, DT_F16 = 1, DT_BF16 = 2 };
+enum { LAY_ROWS = 0, LAY_COLS = 1 };
+
+// ---------------------------------------------------------------------------
+// Plan: radices R0..R{P-1} of the N-point FFT, team size T = N / R0, Q teams per
+// CTA, storage mode of u.
+// ---------------------------------------------------------------------------
+template <int N_, int T_, int Q_, int UMODE_, int MINB_, int... Rs>
+struct Plan {
+  static constexpr int N = N_;
+  static constexpr int MINB = MINB_;  // CTAs per SM the register budget must allow
+  static constexpr int T = T_;
+  static constexpr int Q = Q_;
+  static constexpr int UMODE = UMODE_;
+  static constexpr int NP = sizeof...(Rs);
+  static constexpr int Rv[NP] = {Rs...};
+  static constexpr int E = Rv[0];
+  static constexpr int THREADS = T * Q;
+  static constexpr int NW = (T + 31) / 32;           // warps per team
+  static constexpr int BUF = (N + N / 16 + 8 + 15) / 16 * 16;  // padded float2 slots per team (16-B aligned)
+  static constexpr int RED = 4 * (NW > 1 ? NW : 1);  // float2 reduction slots per team
+  static constexpr size_t SMEM = (size_t)Q * (BUF + RED) * sizeof(float2);
+
+  KD_HD static constexpr int R(int i) { return Rv[i]; }
+  KD_HD static constexpr int B(int i) {  // sub-transform length entering pass i
+    int b = N;
+    for (int j = 0; j < i; ++j) b /= Rv[j];
+    return b;
+  }
+  KD_HD static constexpr bool valid() {
+    int p = 1;
+    for (int i = 0; i < NP; ++i) p *= Rv[i];
+    return p == N && N == T * E && (N % 2 == 0) && NP >= 2 && (T <= 32 ? (32 % T == 0) : (T % 32 == 0 && Q == 1));
+  }
+  static_assert(valid(), "inconsistent plan");
+};
+
+__device__ __forceinline__ int pad(int i) { return i + (i >> 4); }
+
+// Natural index of Makhoul position p (N even).
+template <int N>
+__device__ __forceinline__ int nat_of(int p) {
+  return (p < N / 2) ? 2 * p : 2 * N - 1 - 2 * p;
+}
+
+template <class PL>
+__device__ __forceinline__ void team_sync() {
+  if constexpr (PL::T <= 32) {
+    __syncwarp();
+  } else {
+    __syncthreads();
+  }
+}
+
+// Sum of v over the team; every thread receives the identical result.
+template <class PL>
+__device__ __forceinline__ float2 team_sum(float2 v, float2* red, int lt, int& parity) {
+  constexpr int W = PL::T < 32 ? PL::T : 32;
+#pragma unroll
+  for (int off = W / 2; off > 0; off >>= 1) {
+    v.x = __fadd_rn(v.x, __shfl_xor_sync(0xffffffffu, v.x, off));
+    v.y = __fadd_rn(v.y, __shfl_xor_sync(0xffffffffu, v.y, off));
+  }
+  if constexpr (PL::NW == 1) {
+    return v;
+  } else {
+    float2* r = red + parity * PL::NW;
+    parity ^= 1;
+    if ((lt & 31) == 0) r[lt >> 5] = v;
+    team_sync<PL>();
+    float2 s = r[0];
+#pragma unroll
+    for (int w = 1; w < PL::NW; ++w) s = cadd(s, r[w]);
+    return s;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Radix passes.  tw[j] = exp(-i pi j / N), j < 2N  (W_{2N}^j).
+// Pass i over sub-transforms of length B = B(i): group g -> block g / S, offset
+// np = g % S (S = B / R); elements at block*B + np + j*S.  Forward: radix-R DFT,
+// then twiddle W_B^{np*j} (none on the last pass).  Inverse: conjugate twiddle,
+// then inverse DFT, same slots.
+// ---------------------------------------------------------------------------
+template <class PL, int I, int DIR>
+__device__ __forceinline__ void pass_smem(float2* __restrict__ buf, const float2* __restrict__ tw, int lt) {
+  constexpr int R = PL::R(I);
+  constexpr int Bk = PL::B(I);
+  constexpr int S = Bk / R;
+  constexpr int G = PL::N / R;
+  constexpr bool LAST = (I == PL::NP - 1);
+  constexpr int TWS = 2 * PL::N / Bk;
+  for (int g = lt; g < G; g += PL::T) {
+    const int blk = g / S;
+    const int np = g - blk * S;
+    const int base = blk * Bk + np;
+    float2 v[R];
+#pragma unroll
+    for (int j = 0; j < R; ++j) v[j] = buf[pad(base + j * S)];
+    if constexpr (DIR < 0) {
+      Dft<R, -1>::run(v);
+      if constexpr (!LAST) {
+#pragma unroll
+        for (int j = 1; j < R; ++j) v[j] = cmul(v[j], __ldg(&tw[np * j * TWS]));
+      }
+    } else {
+      if constexpr (!LAST) {
+#pragma unroll
+        for (int j = 1; j < R; ++j) v[j] = cmulc(v[j], __ldg(&tw[np * j * TWS]));
+      }
+      Dft<R, +1>::run(v);
+    }
+#pragma unroll
+    for (int j = 0; j < R; ++j) buf[pad(base + j * S)] = v[j];
+  }
+}
+
+// Digit-reversed slot of frequency k: k = k0 + R0 k1 + R0 R1 k2 + ...  ->
+// slot = k0 (N/R0) + k1 (N/(R0 R1)) + ...
+template <class PL>
+__device__ __forceinline__ int slot_of(int k) {
+  int s = 0;
+  int rem = k;
+  static_for<0, PL::NP>([&](auto ii) {
+    constexpr int I = decltype(ii)::value;
+    constexpr int Ri = PL::R(I);
+    constexpr int stride = PL::B(I) / Ri;
+    const int ki = rem % Ri;
+    rem /= Ri;
+    s += ki * stride;
+  });
+  return s;
+}
+
+__device__ __forceinline__ float eps_of(const uint32_t* __restrict__ eb, int k) {
+  return ((__ldg(&eb[k >> 5]) >> (k & 31)) & 1u) ? -1.f : 1.f;
+}
+
+// The middle operator M (with the 1/N of the inverse DFT folded in).
+template <class PL>
+__device__ __forceinline__ void middle(float2* __restrict__ buf, const float2* __restrict__ tw,
+                                       const uint32_t* __restrict__ eb, int lt) {
+  constexpr int N = PL::N;
+  const float invN = 1.0f / (float)N;
+  for (int i = lt; i <= N / 2; i += PL::T) {
+    if (i == 0 || i == N / 2) {
+      const int s = pad(slot_of<PL>(i));
+      buf[s] = cscale(buf[s], eps_of(eb, i) * invN);
+    } else {
+      const int sa = pad(slot_of<PL>(i));
+      const int sb = pad(slot_of<PL>(N - i));
+      const float2 a = buf[sa];
+      const float2 b = buf[sb];
+      const float ek = eps_of(eb, i);
+      const float ekb = eps_of(eb, N - i);
+      float2 na, nb;
+      if (ek == ekb) {
+        const float f = ek * invN;
+        na = cscale(a, f);
+        nb = cscale(b, f);
+      } else {
+        // w = exp(+i pi k / N) = conj(tw[k]);  Z'_k = ek w Z_{N-k};  Z'_{N-k} = ek conj(w) Z_k
+        const float2 t = __ldg(&tw[i]);
+        const float f = ek * invN;
+        na = cscale(cmulc(b, t), f);
+        nb = cscale(cmul(a, t), f);
+      }
+      buf[sa] = na;
+      buf[sb] = nb;
+    }
+  }
+}
+
+// y = P' v for the team's vector pair held in registers (E values per thread).
+template <class PL>
+__device__ __forceinline__ void apply_P(float2 (&v)[PL::E], float2* __restrict__ buf,
+                                        const float2* __restrict__ tw, const uint32_t* __restrict__ eb,
+                                        int lt) {
+  constexpr int E = PL::E;
+  constexpr int T = PL::T;
+  if constexpr (PL::T <= 32) team_sync<PL>();  // previous readers of buf are done
+  // forward pass 0 from registers: group np = lt, stride T, twiddle W_N^{lt*j} = tw[2*lt*j]
+  Dft<E, -1>::run(v);
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    float2 x = v[j];
+    if (j > 0) x = cmul(x, __ldg(&tw[2 * lt * j]));
+    buf[pad(lt + j * T)] = x;
+  }
+  team_sync<PL>();
+  static_for<1, PL::NP>([&](auto ii) {
+    constexpr int I = decltype(ii)::value;
+    pass_smem<PL, I, -1>(buf, tw, lt);
+    team_sync<PL>();
+  });
+  middle<PL>(buf, tw, eb, lt);
+  team_sync<PL>();
+  static_for<1, PL::NP>([&](auto ii) {
+    constexpr int I = PL::NP - decltype(ii)::value;
+    pass_smem<PL, I, +1>(buf, tw, lt);
+    team_sync<PL>();
+  });
+#pragma unroll
+  for (int j = 0; j < E; ++j) {
+    float2 x = buf[pad(lt + j * T)];
+    if (j > 0) x = cmulc(x, __ldg(&tw[2 * lt * j]));
+    v[j] = x;
+  }
+  Dft<E, +1>::run(v);
+}
+
+// ---------------------------------------------------------------------------
+// Element loads / stores
+// ---------------------------------------------------------------------------
+// dtype and layout are uniform per launch: branching on them costs nothing
+// measurable next to the transform and keeps one kernel per plan.
+__device__ __forceinline__ float load_elem(const void* __restrict__ w, int dt, int64_t idx) {
+  if (dt == DT_F32) return __ldg(reinterpret_cast<const float*>(w) + idx);
+  if (dt == DT_F16) return __half2float(__ldg(reinterpret_cast<const __half*>(w) + idx));
+  return __bfloat162float(__ldg(reinterpret_cast<const __nv_bfloat16*>(w) + idx));
+}
+
+__device__ __forceinline__ void store_elem(void* __restrict__ w, int dt, int64_t idx, float x) {
+  if (dt == DT_F32) {
+    reinterpret_cast<float*>(w)[idx] = x;
+  } else if (dt == DT_F16) {
+    reinterpret_cast<__half*>(w)[idx] = __float2half_rn(x);
+  } else {
+    reinterpret_cast<__nv_bfloat16*>(w)[idx] = __float2bfloat16_rn(x);
+  }
+}
+
+__device__ __forceinline__ int64_t elem_index(int lay, int64_t vec, int i, int64_t ld) {
+  return (lay == LAY_ROWS) ? vec * ld + i : (int64_t)i * ld + vec;
+}
+
+// 2^e as float for -126 <= e <= 127 (exact)
+__device__ __forceinline__ float pow2f(int e) { return __int_as_float((127 + e) << 23); }
+
+// ---------------------------------------------------------------------------
+// Kernel parameters
+// ---------------------------------------------------------------------------
+struct DecParams {
+  const void* w;
+  int dtype, layout;
+  int64_t n, m, ld;
+  int iters;
+  uint32_t* codes_u;
+  uint32_t* codes_v;
+  float* centres_u;
+  float* centres_v;
+  float* coeffs;
+  float* u;
+  float* vhat;
+  float* resid;
+  int8_t* trace;
+  const float2* tw;
+  const uint32_t* eps;
+  uint32_t* status;
+  float2* uslots;
+  int64_t npairs;
+};
+
+// sign(r) * c with sign(0) = 0
+__device__ __forceinline__ float signed_step(float r, float c) {
+  return (r == 0.f) ? 0.f : copysignf(c, r);
+}
+
+// ---------------------------------------------------------------------------
+// kd_decompose kernel
+// ---------------------------------------------------------------------------
+template <class PL>
+__global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecParams p) {
+  constexpr int N = PL::N;
+  constexpr int T = PL::T;
+  constexpr int E = PL::E;
+  extern __shared__ __align__(16) float2 smem[];
+  const int team = threadIdx.x / T;
+  const int lt = threadIdx.x - team * T;
+  float2* buf = smem + team * (PL::BUF + PL::RED);
+  float2* red = buf + PL::BUF;
+  int parity = 0;
+  const int nsteps = 4 * p.iters;
+
+  float2 uu_reg[PL::UMODE == UREG ? E : 1];
+  float2* uslot = nullptr;
+  if constexpr (PL::UMODE == UGMEM) uslot = p.uslots + ((int64_t)blockIdx.x * PL::Q + team) * N;
+
+  for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
+    const int64_t pair = base + team;
+    const bool active = pair < p.npairs;
+    const int64_t pr = active ? pair : base;
+    const int64_t colA = 2 * pr;
+    const bool hasB = (colA + 1) < p.m;
+    const int64_t colB = hasB ? colA + 1 : colA;
+
+    // ---- load the pair in Makhoul order: position lt + j*T ----
+    float2 r[E];
+    float2 acc = make_float2(0.f, 0.f);
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      const int nat = nat_of<N>(lt + j * T);
+      const float a = load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld));
+      const float b = hasB ? load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)) : 0.f;
+      r[j] = make_float2(a, b);
+      acc.x = __fadd_rn(acc.x, fabsf(a));
+      acc.y = __fadd_rn(acc.y, fabsf(b));
+    }
+    float2 sum0 = team_sum<PL>(acc, red, lt, parity);
+    // ---- exact power-of-two normalisation: c1 of each vector lands in [1, 2) ----
+    int sA = 0, sB = 0;
+    {
+      const bool finA = isfinite(sum0.x), finB = isfinite(sum0.y);
+      if (active && lt == 0 && (!finA || !finB)) atomicOr(p.status, 1u);
+      const float cA = __fdiv_rn(sum0.x, (float)N), cB = __fdiv_rn(sum0.y, (float)N);
+      if (finA && cA > 0.f) sA = max(-100, min(100, -ilogbf(cA)));
+      if (finB && cB > 0.f) sB = max(-100, min(100, -ilogbf(cB)));
+    }
+    const float scA = pow2f(sA), scB = pow2f(sB);
+#pragma unroll
+    for (int j = 0; j < E; ++j) r[j] = make_float2(__fmul_rn(r[j].x, scA), __fmul_rn(r[j].y, scB));
+    sum0 = make_float2(__fmul_rn(sum0.x, scA), __fmul_rn(sum0.y, scB));
+
+    if constexpr (PL::UMODE == UREG) {
+#pragma unroll
+      for (int j = 0; j < E; ++j) uu_reg[j] = make_float2(0.f, 0.f);
+    } else {
+#pragma unroll
+      for (int j = 0; j < E; ++j) uslot[lt + j * T] = make_float2(0.f, 0.f);
+    }
+    float2 coef[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) coef[q] = make_float2(0.f, 0.f);
+
+    const bool tracing = (p.trace != nullptr) && active;
+    int8_t* trA = nullptr;
+    int8_t* trB = nullptr;
+    if (tracing) {
+      trA = p.trace + colA * (int64_t)nsteps * N;
+      trB = p.trace + colB * (int64_t)nsteps * N;
+    }
+
+    // One atomic greedy step on the values in r: lambda = ||r||_1 / N per vector,
+    // r -= sign(r) lambda; the applied step is returned through `add` callback.
+    auto greedy = [&](int step, bool have_sum, float2 presum, auto&& add) -> float2 {
+      float2 s = presum;
+      if (!have_sum) {
+        float2 a = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < E; ++j) {
+          a.x = __fadd_rn(a.x, fabsf(r[j].x));
+          a.y = __fadd_rn(a.y, fabsf(r[j].y));
+        }
+        s = team_sum<PL>(a, red, lt, parity);
+      }
+      const float lA = __fdiv_rn(s.x, (float)N);
+      const float lB = __fdiv_rn(s.y, (float)N);
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        if (tracing) {
+          const int nat = nat_of<N>(lt + j * T);
+          const int64_t off = (int64_t)step * N + nat;
+          trA[off] = (int8_t)((r[j].x > 0.f) - (r[j].x < 0.f));
+          if (hasB) trB[off] = (int8_t)((r[j].y > 0.f) - (r[j].y < 0.f));
+        }
+        const float dA = signed_step(r[j].x, lA);
+        const float dB = signed_step(r[j].y, lB);
+        r[j].x = __fsub_rn(r[j].x, dA);
+        r[j].y = __fsub_rn(r[j].y, dB);
+        add(j, dA, dB);
+      }
+      return make_float2(lA, lB);
+    };
+    auto add_u = [&](int j, float dA, float dB) {
+      if constexpr (PL::UMODE == UREG) {
+        uu_reg[j].x = __fadd_rn(uu_reg[j].x, dA);
+        uu_reg[j].y = __fadd_rn(uu_reg[j].y, dB);
+      }
+    };
+    auto add_none = [&](int, float, float) {};
+
+    int step = 0;
+    for (int t = 0; t < p.iters; ++t) {
+      // two greedy steps from Q_N (update u)
+      float2 ugm[PL::UMODE == UGMEM ? E : 1];
+      if constexpr (PL::UMODE == UGMEM) {
+#pragma unroll
+        for (int j = 0; j < E; ++j) ugm[j] = uslot[lt + j * T];
+      }
+      auto add_u_any = [&](int j, float dA, float dB) {
+        if constexpr (PL::UMODE == UREG) {
+          add_u(j, dA, dB);
+        } else {
+          ugm[j].x = __fadd_rn(ugm[j].x, dA);
+          ugm[j].y = __fadd_rn(ugm[j].y, dB);
+        }
+      };
+      float2 l1 = greedy(step, t == 0, sum0, add_u_any);
+      ++step;
+      float2 l2 = greedy(step, false, sum0, add_u_any);
+      ++step;
+      if constexpr (PL::UMODE == UGMEM) {
+#pragma unroll
+        for (int j = 0; j < E; ++j) uslot[lt + j * T] = ugm[j];
+      }
+      // two greedy steps from P Q_N on y = P rho (update vhat implicitly)
+      apply_P<PL>(r, buf, p.tw, p.eps, lt);
+      float2 l3 = greedy(step, false, sum0, add_none);
+      ++step;
+      float2 l4 = greedy(step, false, sum0, add_none);
+      ++step;
+      apply_P<PL>(r, buf, p.tw, p.eps, lt);
+      if (t == 0) {
+        coef[0] = l1;
+        coef[1] = l2;
+        coef[2] = l3;
+        coef[3] = l4;
+      }
+    }
+
+    // ---- vhat = P (x - u - r) ----
+    float2 vh[E];
+    float2 uf[E];
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      const int nat = nat_of<N>(lt + j * T);
+      const float a = __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld)), scA);
+      const float b = hasB ? __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)), scB) : 0.f;
+      if constexpr (PL::UMODE == UREG) {
+        uf[j] = uu_reg[j];
+      } else {
+        uf[j] = uslot[lt + j * T];
+      }
+      vh[j] = make_float2(__fsub_rn(__fsub_rn(a, uf[j].x), r[j].x), __fsub_rn(__fsub_rn(b, uf[j].y), r[j].y));
+    }
+    if (p.iters > 0) {
+      apply_P<PL>(vh, buf, p.tw, p.eps, lt);
+    } else {
+#pragma unroll
+      for (int j = 0; j < E; ++j) vh[j] = make_float2(0.f, 0.f);
+    }
+
+    // ---- optional dense outputs (natural order, scaled back) ----
+    const float isA = pow2f(-sA), isB = pow2f(-sB);
+    if (active) {
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        const int nat = nat_of<N>(lt + j * T);
+        if (p.u) {
+          p.u[colA * N + nat] = __fmul_rn(uf[j].x, isA);
+          if (hasB) p.u[colB * N + nat] = __fmul_rn(uf[j].y, isB);
+        }
+        if (p.vhat) {
+          p.vhat[colA * N + nat] = __fmul_rn(vh[j].x, isA);
+          if (hasB) p.vhat[colB * N + nat] = __fmul_rn(vh[j].y, isB);
+        }
+        if (p.resid) {
+          p.resid[colA * N + nat] = __fmul_rn(r[j].x, isA);
+          if (hasB) p.resid[colB * N + nat] = __fmul_rn(r[j].y, isB);
+        }
+      }
+    }
+
+    // ---- 2-bit codes: nearest of the closed-form centres, ties low ----
+    const float muA = fmaxf(coef[0].x, coef[1].x), muB = fmaxf(coef[0].y, coef[1].y);
+    const float mvA = fmaxf(coef[2].x, coef[3].x), mvB = fmaxf(coef[2].y, coef[3].y);
+    team_sync<PL>();  // everyone is done with buf
+    uint8_t* cb = reinterpret_cast<uint8_t*>(buf);
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      const int nat = nat_of<N>(lt + j * T);
+      auto code = [](float x, float mm) -> uint8_t {
+        return (uint8_t)((x > -mm) + (x > 0.f) + (x > mm));
+      };
+      cb[0 * N + nat] = code(uf[j].x, muA);
+      cb[1 * N + nat] = code(uf[j].y, muB);
+      cb[2 * N + nat] = code(vh[j].x, mvA);
+      cb[3 * N + nat] = code(vh[j].y, mvB);
+    }
+    team_sync<PL>();
+    constexpr int WPV = N / 16;  // words per vector (N % 16 == 0 for every plan)
+    static_assert(N % 16 == 0, "plans keep N a multiple of 16");
+    if (active) {
+      for (int wi = lt; wi < 4 * WPV; wi += T) {
+        const int plane = wi / WPV;
+        const int word = wi - plane * WPV;
+        const uint4 q = *reinterpret_cast<const uint4*>(cb + plane * N + word * 16);
+        const uint32_t qq[4] = {q.x, q.y, q.z, q.w};
+        uint32_t packed = 0;
+#pragma unroll
+        for (int b4 = 0; b4 < 4; ++b4) {
+#pragma unroll
+          for (int by = 0; by < 4; ++by) packed |= ((qq[b4] >> (8 * by)) & 3u) << (2 * (4 * b4 + by));
+        }
+        const bool isB = (plane & 1) != 0;
+        if (isB && !hasB) continue;
+        const int64_t col = isB ? colB : colA;
+        uint32_t* dst = (plane < 2) ? p.codes_u : p.codes_v;
+        dst[col * WPV + word] = packed;
+      }
+      if (lt == 0) {
+        const float sc[2] = {isA, isB};
+        for (int v2 = 0; v2 < (hasB ? 2 : 1); ++v2) {
+          const int64_t col = v2 ? colB : colA;
+          const float c1 = v2 ? coef[0].y : coef[0].x, c2 = v2 ? coef[1].y : coef[1].x;
+          const float d1 = v2 ? coef[2].y : coef[2].x, d2 = v2 ? coef[3].y : coef[3].x;
+          const float f = sc[v2];
+          const float uo = __fmul_rn(__fadd_rn(c1, c2), f), ui = __fmul_rn(fabsf(__fsub_rn(c1, c2)), f);
+          const float vo = __fmul_rn(__fadd_rn(d1, d2), f), vi = __fmul_rn(fabsf(__fsub_rn(d1, d2)), f);
+          float* cu = p.centres_u + col * 4;
+          float* cv = p.centres_v + col * 4;
+          cu[0] = -uo; cu[1] = -ui; cu[2] = ui; cu[3] = uo;
+          cv[0] = -vo; cv[1] = -vi; cv[2] = vi; cv[3] = vo;
+          if (p.coeffs) {
+            float* co = p.coeffs + col * 4;
+            co[0] = __fmul_rn(c1, f); co[1] = __fmul_rn(c2, f);
+            co[2] = __fmul_rn(d1, f); co[3] = __fmul_rn(d2, f);
+          }
+        }
+      }
+    }
+    team_sync<PL>();  // buf is reused by the next pair
+  }
+}
+
+// ---------------------------------------------------------------------------
+// kd_apply_p kernel: y_j = P x_j, fp32 vector-major.
+// ---------------------------------------------------------------------------
+struct ApplyParams {
+  const float* x;
+  float* y;
+  int64_t m;
+  const float2* tw;
+  const uint32_t* eps;
+  int64_t npairs;
+};
+
+template <class PL>
+__global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyParams p) {
+  constexpr int N = PL::N;
+  constexpr int T = PL::T;
+  constexpr int E = PL::E;
+  extern __shared__ __align__(16) float2 smem[];
+  const int team = threadIdx.x / T;
+  const int lt = threadIdx.x - team * T;
+  float2* buf = smem + team * (PL::BUF + PL::RED);
+  for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
+    const int64_t pair = base + team;
+    const bool active = pair < p.npairs;
+    const int64_t pr = active ? pair : base;
+    const int64_t colA = 2 * pr;
+    const bool hasB = (colA + 1) < p.m;
+    float2 v[E];
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      const int nat = nat_of<N>(lt + j * T);
+      v[j] = make_float2(__ldg(&p.x[colA * N + nat]), hasB ? __ldg(&p.x[(colA + 1) * N + nat]) : 0.f);
+    }
+    team_sync<PL>();  // x and y may alias: all loads of this pair precede any store
+    apply_P<PL>(v, buf, p.tw, p.eps, lt);
+    if (active) {
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        const int nat = nat_of<N>(lt + j * T);
+        p.y[colA * N + nat] = v[j].x;
+        if (hasB) p.y[(colA + 1) * N + nat] = v[j].y;
+      }
+    }
+    team_sync<PL>();
+  }
+}
+
+// ---------------------------------------------------------------------------
+// kd_reconstruct kernel: W_hat_j = cu_j[code_u] + P(cv_j[code_v])   (App. C)
+// ---------------------------------------------------------------------------
+struct RecParams {
+  int dtype, layout;
+  const uint32_t* codes_u;
+  const uint32_t* codes_v;
+  const float* centres_u;
+  const float* centres_v;
+  int64_t m, ld;
+  void* out;
+  const float2* tw;
+  const uint32_t* eps;
+  int64_t npairs;
+};
+
+template <class PL>
+__global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecParams p) {
+  constexpr int N = PL::N;
+  constexpr int T = PL::T;
+  constexpr int E = PL::E;
+  constexpr int WPV = N / 16;
+  extern __shared__ __align__(16) float2 smem[];
+  const int team = threadIdx.x / T;
+  const int lt = threadIdx.x - team * T;
+  float2* buf = smem + team * (PL::BUF + PL::RED);
+  for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
+    const int64_t pair = base + team;
+    const bool active = pair < p.npairs;
+    const int64_t pr = active ? pair : base;
+    const int64_t colA = 2 * pr;
+    const bool hasB = (colA + 1) < p.m;
+    const int64_t colB = hasB ? colA + 1 : colA;
+    float2 uq[E], vq[E];
+#pragma unroll
+    for (int j = 0; j < E; ++j) {
+      const int nat = nat_of<N>(lt + j * T);
+      const int word = nat >> 4, sh = 2 * (nat & 15);
+      const int cuA = (__ldg(&p.codes_u[colA * WPV + word]) >> sh) & 3;
+      const int cvA = (__ldg(&p.codes_v[colA * WPV + word]) >> sh) & 3;
+      float ua = __ldg(&p.centres_u[colA * 4 + cuA]);
+      float va = __ldg(&p.centres_v[colA * 4 + cvA]);
+      float ub = 0.f, vb = 0.f;
+      if (hasB) {
+        const int cuB = (__ldg(&p.codes_u[colB * WPV + word]) >> sh) & 3;
+        const int cvB = (__ldg(&p.codes_v[colB * WPV + word]) >> sh) & 3;
+        ub = __ldg(&p.centres_u[colB * 4 + cuB]);
+        vb = __ldg(&p.centres_v[colB * 4 + cvB]);
+      }
+      uq[j] = make_float2(ua, ub);
+      vq[j] = make_float2(va, vb);
+    }
+    apply_P<PL>(vq, buf, p.tw, p.eps, lt);
+    if (active) {
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        const int nat = nat_of<N>(lt + j * T);
+        store_elem(p.out, p.dtype, elem_index(p.layout, colA, nat, p.ld), __fadd_rn(uq[j].x, vq[j].x));
+        if (hasB) store_elem(p.out, p.dtype, elem_index(p.layout, colB, nat, p.ld), __fadd_rn(uq[j].y, vq[j].y));
+      }
+    }
+    team_sync<PL>();
+  }
+}
+
+}  // namespace kd

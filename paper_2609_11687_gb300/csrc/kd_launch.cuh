@@ -1,0 +1,64 @@
+// Launch helpers shared by the per-N translation units.
+#pragma once
+#include <mutex>
+
+#include "kd_kernels.cuh"
+#include "kd_ops.h"
+
+namespace kd {
+
+template <class K>
+inline cudaError_t prepare(K kernel, size_t smem) {
+  // Opt in to more than 48 KB of dynamic shared memory, once per kernel.
+  static std::once_flag once;
+  static cudaError_t err = cudaSuccess;
+  std::call_once(once, [&] {
+    err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  });
+  return err;
+}
+
+template <class K>
+inline int occupancy(K kernel, int threads, size_t smem) {
+  if (prepare(kernel, smem) != cudaSuccess) return 0;
+  int nb = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kernel, threads, smem) != cudaSuccess) return 0;
+  return nb;
+}
+
+template <class PL>
+struct Ops {
+  static cudaError_t decompose(const DecParams& p, int grid, cudaStream_t s) {
+    auto k = decompose_kernel<PL>;
+    cudaError_t e = prepare(k, PL::SMEM);
+    if (e != cudaSuccess) return e;
+    k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
+    return cudaGetLastError();
+  }
+  static cudaError_t reconstruct(const RecParams& p, int grid, cudaStream_t s) {
+    auto k = reconstruct_kernel<PL>;
+    cudaError_t e = prepare(k, PL::SMEM);
+    if (e != cudaSuccess) return e;
+    k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
+    return cudaGetLastError();
+  }
+  static cudaError_t apply(const ApplyParams& p, int grid, cudaStream_t s) {
+    auto k = apply_p_kernel<PL>;
+    cudaError_t e = prepare(k, PL::SMEM);
+    if (e != cudaSuccess) return e;
+    k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
+    return cudaGetLastError();
+  }
+  static int ctas_per_sm(int which) {
+    if (which == 0) return occupancy(decompose_kernel<PL>, PL::THREADS, PL::SMEM);
+    if (which == 1) return occupancy(apply_p_kernel<PL>, PL::THREADS, PL::SMEM);
+    return occupancy(reconstruct_kernel<PL>, PL::THREADS, PL::SMEM);
+  }
+  static const PlanOps* ops() {
+    static const PlanOps o{PL::N, PL::THREADS, PL::Q, PL::SMEM, PL::UMODE == UGMEM,
+                           &Ops::ctas_per_sm, &Ops::decompose, &Ops::apply, &Ops::reconstruct};
+    return &o;
+  }
+};
+
+}  // namespace kd

@@ -1,0 +1,277 @@
+// Device arithmetic for the Kashin-DCT kernels: complex helpers, compile-time
+// trigonometric constants, and in-register small DFTs.
+//
+// All floating-point operations here use explicit round-to-nearest intrinsics
+// (the library is compiled with --fmad=false), so every instantiation of a kernel
+// performs the same operations in the same order: the trace build and the
+// timed build are bitwise identical.
+#pragma once
+
+#include <cstdint>
+#include <type_traits>
+#include <cuda_runtime.h>
+
+#define KD_HD __host__ __device__
+
+namespace kd {
+
+// ---------------------------------------------------------------------------
+// Compile-time cos / sin of 2*pi*a/b (double), from the Taylor series after an
+// exact rational reduction of the angle to [-pi/4, pi/4].
+// ---------------------------------------------------------------------------
+constexpr double kPi = 3.141592653589793238462643383279502884;
+
+KD_HD constexpr double taylor_sin(double x) {
+  double term = x, sum = x;
+  for (int k = 1; k < 16; ++k) {
+    term *= -x * x / ((2.0 * k) * (2.0 * k + 1.0));
+    sum += term;
+  }
+  return sum;
+}
+
+KD_HD constexpr double taylor_cos(double x) {
+  double term = 1.0, sum = 1.0;
+  for (int k = 1; k < 16; ++k) {
+    term *= -x * x / ((2.0 * k - 1.0) * (2.0 * k));
+    sum += term;
+  }
+  return sum;
+}
+
+// angle 2*pi*a/b: a reduced mod b, q = nearest quarter turn, remainder exact.
+KD_HD constexpr long long kd_mod(long long a, long long b) { return ((a % b) + b) % b; }
+
+KD_HD constexpr double cos2pi(long long a, long long b) {
+  long long r = kd_mod(a, b);
+  long long q = (4 * r * 2 + b) / (2 * b);  // round(4r/b)
+  double f = kPi * (double)(4 * r - q * b) / (2.0 * (double)b);
+  switch (q & 3) {
+    case 0: return taylor_cos(f);
+    case 1: return -taylor_sin(f);
+    case 2: return -taylor_cos(f);
+    default: return taylor_sin(f);
+  }
+}
+
+KD_HD constexpr double sin2pi(long long a, long long b) {
+  long long r = kd_mod(a, b);
+  long long q = (4 * r * 2 + b) / (2 * b);
+  double f = kPi * (double)(4 * r - q * b) / (2.0 * (double)b);
+  switch (q & 3) {
+    case 0: return taylor_sin(f);
+    case 1: return taylor_cos(f);
+    case 2: return -taylor_sin(f);
+    default: return -taylor_cos(f);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Complex helpers (float2 = re, im)
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float2 cadd(float2 a, float2 b) {
+  return make_float2(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y));
+}
+__device__ __forceinline__ float2 csub(float2 a, float2 b) {
+  return make_float2(__fsub_rn(a.x, b.x), __fsub_rn(a.y, b.y));
+}
+// a * b
+__device__ __forceinline__ float2 cmul(float2 a, float2 b) {
+  return make_float2(__fmaf_rn(a.x, b.x, __fmul_rn(-a.y, b.y)),
+                     __fmaf_rn(a.x, b.y, __fmul_rn(a.y, b.x)));
+}
+// a * conj(b)
+__device__ __forceinline__ float2 cmulc(float2 a, float2 b) {
+  return make_float2(__fmaf_rn(a.x, b.x, __fmul_rn(a.y, b.y)),
+                     __fmaf_rn(a.y, b.x, __fmul_rn(-a.x, b.y)));
+}
+__device__ __forceinline__ float2 cscale(float2 a, float s) {
+  return make_float2(__fmul_rn(a.x, s), __fmul_rn(a.y, s));
+}
+// -i * a   (exact)
+__device__ __forceinline__ float2 mul_mi(float2 a) { return make_float2(a.y, -a.x); }
+// +i * a   (exact)
+__device__ __forceinline__ float2 mul_pi(float2 a) { return make_float2(-a.y, a.x); }
+
+// Multiply by the compile-time root W_R^E = exp(DIR * 2 pi i E / R), DIR = -1 forward.
+// Quarter turns are exact; eighth turns use one constant; others a full product.
+template <int DIR, long long E, long long R>
+__device__ __forceinline__ float2 mul_root(float2 a) {
+  constexpr long long e = kd_mod(E, R);
+  if constexpr (e == 0) {
+    return a;
+  } else if constexpr ((4 * e) % R == 0) {
+    constexpr long long qtr = (4 * e) / R;  // 1, 2, 3 quarter turns (counter-clockwise for DIR=+1)
+    constexpr long long q = (DIR > 0) ? qtr : (4 - qtr) % 4;
+    if constexpr (q == 1) return mul_pi(a);
+    else if constexpr (q == 2) return make_float2(-a.x, -a.y);
+    else return mul_mi(a);
+  } else if constexpr ((8 * e) % R == 0) {
+    constexpr float h = (float)0.70710678118654752440084436210484903928;
+    constexpr long long o = (8 * e) / R;  // odd octant 1,3,5,7
+    constexpr long long oo = (DIR > 0) ? o : (8 - o);
+    // exp(i*pi*oo/4) = (c, s) with |c| = |s| = h
+    constexpr float c = (oo == 1 || oo == 7) ? h : -h;
+    constexpr float s = (oo == 1 || oo == 3) ? h : -h;
+    // (a.x + i a.y)(c + i s) = (c a.x - s a.y) + i (s a.x + c a.y)
+    // c*(a.x - (s/c) a.y), c*(a.y + (s/c) a.x) with s/c = +-1 exact
+    if constexpr ((c > 0) == (s > 0)) {
+      return make_float2(__fmul_rn(c, __fsub_rn(a.x, a.y)), __fmul_rn(c, __fadd_rn(a.y, a.x)));
+    } else {
+      return make_float2(__fmul_rn(c, __fadd_rn(a.x, a.y)), __fmul_rn(c, __fsub_rn(a.y, a.x)));
+    }
+  } else {
+    constexpr float c = (float)cos2pi(e, R);
+    constexpr float s = (float)((DIR > 0 ? 1.0 : -1.0) * sin2pi(e, R));
+    return make_float2(__fmaf_rn(a.x, c, __fmul_rn(-a.y, s)), __fmaf_rn(a.x, s, __fmul_rn(a.y, c)));
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Compile-time loop: f(std::integral_constant<int, I>{}) for I in [B, E).
+// ---------------------------------------------------------------------------
+template <int I>
+using ic = std::integral_constant<int, I>;
+
+template <int B, int E, class F>
+__device__ __forceinline__ void static_for(F&& f) {
+  if constexpr (B < E) {
+    f(ic<B>{});
+    static_for<B + 1, E>(f);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// In-register DFT of size R (DIR = -1 forward, +1 inverse, unnormalised):
+//   X[k] = sum_n x[n] exp(DIR * 2 pi i n k / R), natural order in and out.
+// ---------------------------------------------------------------------------
+template <int R>
+struct SmallestFactor {
+  static constexpr int value = (R % 4 == 0 && R > 4) ? 4 : (R % 2 == 0) ? 2 : (R % 3 == 0) ? 3
+                             : (R % 5 == 0) ? 5 : (R % 7 == 0) ? 7 : R;
+};
+
+template <int R, int DIR>
+struct Dft;
+
+template <int DIR>
+struct Dft<1, DIR> {
+  template <class A>
+  __device__ __forceinline__ static void run(A&) {}
+};
+
+template <int DIR>
+struct Dft<2, DIR> {
+  template <class A>
+  __device__ __forceinline__ static void run(A& v) {
+    float2 a = v[0], b = v[1];
+    v[0] = cadd(a, b);
+    v[1] = csub(a, b);
+  }
+};
+
+template <int DIR>
+struct Dft<4, DIR> {
+  template <class A>
+  __device__ __forceinline__ static void run(A& v) {
+    float2 s02 = cadd(v[0], v[2]), d02 = csub(v[0], v[2]);
+    float2 s13 = cadd(v[1], v[3]), d13 = csub(v[1], v[3]);
+    // forward: X1 = d02 - i d13, X3 = d02 + i d13 ; inverse: signs swapped
+    float2 t = (DIR < 0) ? mul_mi(d13) : mul_pi(d13);
+    v[0] = cadd(s02, s13);
+    v[2] = csub(s02, s13);
+    v[1] = cadd(d02, t);
+    v[3] = csub(d02, t);
+  }
+};
+
+// Odd prime R: symmetric direct form.  a_n = x_n + x_{R-n}, b_n = x_n - x_{R-n};
+// X_k = x_0 + sum a_n cos(2 pi n k / R) -+ i sum b_n sin(2 pi n k / R).
+template <int R, int DIR>
+struct DftPrime {
+  template <class Arr>
+  __device__ __forceinline__ static void run(Arr& v) {
+    constexpr int H = (R - 1) / 2;
+    float2 a[H + 1], b[H + 1];
+    const float2 x0 = v[0];
+    float2 sum = x0;
+#pragma unroll
+    for (int n = 1; n <= H; ++n) {
+      a[n] = cadd(v[n], v[R - n]);
+      b[n] = csub(v[n], v[R - n]);
+      sum = cadd(sum, a[n]);
+    }
+    v[0] = sum;
+    static_for<1, H + 1>([&](auto kk) {
+      constexpr int K = decltype(kk)::value;
+      float2 ak = x0;
+      float2 bk = make_float2(0.f, 0.f);
+      static_for<1, H + 1>([&](auto nn) {
+        constexpr int NN = decltype(nn)::value;
+        constexpr float c = (float)cos2pi((long long)NN * K, R);
+        constexpr float s = (float)sin2pi((long long)NN * K, R);
+        ak.x = __fmaf_rn(a[NN].x, c, ak.x);
+        ak.y = __fmaf_rn(a[NN].y, c, ak.y);
+        bk.x = __fmaf_rn(b[NN].x, s, bk.x);
+        bk.y = __fmaf_rn(b[NN].y, s, bk.y);
+      });
+      // forward: X_k = ak - i bk, X_{R-k} = ak + i bk ; inverse: the reverse
+      const float2 ib = mul_pi(bk);
+      if constexpr (DIR < 0) {
+        v[K] = csub(ak, ib);
+        v[R - K] = cadd(ak, ib);
+      } else {
+        v[K] = cadd(ak, ib);
+        v[R - K] = csub(ak, ib);
+      }
+    });
+  }
+};
+
+// Composite R = A * B (A = smallest factor, 4 preferred): decimation in frequency.
+//   n = B*n1 + n2 ; k = k1 + A*k2
+//   step 1: for each n2, size-A DFT over n1 -> k1 ; multiply by W_R^{n2*k1}
+//   step 2: for each k1, size-B DFT over n2 -> k2.
+template <int R, int DIR>
+struct DftComposite {
+  static constexpr int A = SmallestFactor<R>::value;
+  static constexpr int B = R / A;
+  template <class Arr>
+  __device__ __forceinline__ static void run(Arr& v) {
+    float2 t[R];
+    static_for<0, B>([&](auto n2c) {
+      constexpr int N2 = decltype(n2c)::value;
+      float2 s[A];
+#pragma unroll
+      for (int n1 = 0; n1 < A; ++n1) s[n1] = v[B * n1 + N2];
+      Dft<A, DIR>::run(s);
+      static_for<0, A>([&](auto k1c) {
+        constexpr int K1 = decltype(k1c)::value;
+        t[K1 * B + N2] = mul_root<DIR, (long long)N2 * K1, R>(s[K1]);
+      });
+    });
+#pragma unroll
+    for (int k1 = 0; k1 < A; ++k1) {
+      float2 s[B];
+#pragma unroll
+      for (int n2 = 0; n2 < B; ++n2) s[n2] = t[k1 * B + n2];
+      Dft<B, DIR>::run(s);
+#pragma unroll
+      for (int k2 = 0; k2 < B; ++k2) v[k1 + A * k2] = s[k2];
+    }
+  }
+};
+
+template <int R, int DIR>
+struct Dft {
+  template <class A>
+  __device__ __forceinline__ static void run(A& v) {
+    if constexpr (SmallestFactor<R>::value == R) {
+      DftPrime<R, DIR>::run(v);
+    } else {
+      DftComposite<R, DIR>::run(v);
+    }
+  }
+};
+
+}  // namespace kd

@@ -1,0 +1,27 @@
+// Host-side interface between the C ABI (kd_api.cu) and the per-N translation
+// units (kd_plan_<N>.cu), each of which instantiates the kernels of one plan.
+#pragma once
+#include <cstddef>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace kd {
+struct DecParams;
+struct ApplyParams;
+struct RecParams;
+
+struct PlanOps {
+  int n;
+  int threads;      // threads per CTA
+  int q;            // vector pairs per CTA per iteration
+  size_t smem;      // dynamic shared memory per CTA
+  bool u_in_gmem;   // u lives in per-team workspace slots
+  // CTAs that fit on one SM (occupancy), 0 on error
+  int (*ctas_per_sm)(int which);  // which: 0 decompose, 1 apply, 2 reconstruct
+  cudaError_t (*decompose)(const DecParams&, int grid, cudaStream_t);
+  cudaError_t (*apply)(const ApplyParams&, int grid, cudaStream_t);
+  cudaError_t (*reconstruct)(const RecParams&, int grid, cudaStream_t);
+};
+
+const PlanOps* plan_ops(int64_t n);
+}  // namespace kd

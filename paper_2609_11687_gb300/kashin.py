@@ -1,0 +1,267 @@
+"""Python binding of libkashin (include/kashin.h).
+
+Argument marshalling only: device memory comes from PyTorch tensors, streams
+from ``torch.cuda``; every step of the decomposition, coding, transform and
+reconstruction runs in the library's CUDA kernels.  Importing this module loads
+``libkashin.so`` from this package directory and raises ``ImportError`` if it is
+missing -- there is no fallback implementation.
+
+Two layers:
+
+* ``kd_*`` functions mirror the C entry points one to one (raw device pointers
+  as Python ints, a status code back);
+* ``decompose`` / ``apply_p`` / ``reconstruct`` take and return torch tensors.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import Optional
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libkashin.so")
+
+KD_OK, KD_ERR_INVALID_ARG, KD_ERR_UNSUPPORTED_N, KD_ERR_CUDA, KD_ERR_NONFINITE, KD_ERR_WORKSPACE = range(6)
+KD_F32, KD_F16, KD_BF16 = 0, 1, 2
+KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
+
+EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
+           "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status")
+
+
+def _load() -> ctypes.CDLL:
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is not built; run paper_2609_11687_gb300.build.build() "
+                          "(the CUDA library is required, there is no CPU fallback)")
+    lib = ctypes.CDLL(LIB_PATH)
+    c_i64, c_u64, c_int, c_vp, c_sz = ctypes.c_int64, ctypes.c_uint64, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t
+    lib.kd_status_string.argtypes = [c_int]
+    lib.kd_status_string.restype = ctypes.c_char_p
+    lib.kd_version.argtypes = []
+    lib.kd_version.restype = ctypes.c_char_p
+    lib.kd_supported.argtypes = [c_i64]
+    lib.kd_supported.restype = c_int
+    lib.kd_workspace_size.argtypes = [c_i64]
+    lib.kd_workspace_size.restype = c_sz
+    lib.kd_signs.argtypes = [c_u64, c_i64, c_vp]
+    lib.kd_signs.restype = c_int
+    lib.kd_decompose.argtypes = [c_vp, c_int, c_int, c_i64, c_i64, c_i64, c_u64, c_int,
+                                 c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_sz, c_vp]
+    lib.kd_decompose.restype = c_int
+    lib.kd_apply_p.argtypes = [c_vp, c_vp, c_i64, c_i64, c_u64, c_vp, c_sz, c_vp]
+    lib.kd_apply_p.restype = c_int
+    lib.kd_reconstruct.argtypes = [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_u64, c_int, c_int, c_vp,
+                                   c_i64, c_vp, c_sz, c_vp]
+    lib.kd_reconstruct.restype = c_int
+    lib.kd_read_status.argtypes = [c_vp, c_vp]
+    lib.kd_read_status.restype = c_int
+    return lib
+
+
+lib = _load()
+
+
+class KashinError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {status_string(status)}")
+
+
+def status_string(s: int) -> str:
+    return lib.kd_status_string(int(s)).decode()
+
+
+def version() -> str:
+    return lib.kd_version().decode()
+
+
+# ---------------------------------------------------------------------------
+# one-to-one mirrors of the C entry points
+# ---------------------------------------------------------------------------
+
+def kd_supported(n: int) -> int:
+    return lib.kd_supported(int(n))
+
+
+def kd_workspace_size(n: int) -> int:
+    return int(lib.kd_workspace_size(int(n)))
+
+
+def kd_signs(sign_seed: int, n: int) -> np.ndarray:
+    out = np.empty(int(n), dtype=np.int8)
+    st = lib.kd_signs(ctypes.c_uint64(int(sign_seed) & ((1 << 64) - 1)), int(n), out.ctypes.data)
+    if st != KD_OK:
+        raise KashinError(st, "kd_signs")
+    return out
+
+
+def kd_decompose(w, dtype, layout, n, m, ld, sign_seed, iters, codes_u, codes_v, centres_u, centres_v,
+                 coeffs, u, vhat, resid, trace, workspace, ws_bytes, stream) -> int:
+    return lib.kd_decompose(w, dtype, layout, n, m, ld, ctypes.c_uint64(int(sign_seed) & ((1 << 64) - 1)),
+                            iters, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat, resid, trace,
+                            workspace, ws_bytes, stream)
+
+
+def kd_apply_p(x, y, n, m, sign_seed, workspace, ws_bytes, stream) -> int:
+    return lib.kd_apply_p(x, y, n, m, ctypes.c_uint64(int(sign_seed) & ((1 << 64) - 1)), workspace, ws_bytes,
+                          stream)
+
+
+def kd_reconstruct(codes_u, codes_v, centres_u, centres_v, n, m, sign_seed, out_dtype, layout, w_hat, ld,
+                   workspace, ws_bytes, stream) -> int:
+    return lib.kd_reconstruct(codes_u, codes_v, centres_u, centres_v, n, m,
+                              ctypes.c_uint64(int(sign_seed) & ((1 << 64) - 1)), out_dtype, layout, w_hat, ld,
+                              workspace, ws_bytes, stream)
+
+
+def kd_read_status(workspace, stream) -> int:
+    return lib.kd_read_status(workspace, stream)
+
+
+# ---------------------------------------------------------------------------
+# torch-tensor wrappers
+# ---------------------------------------------------------------------------
+
+def _torch():
+    import torch
+    return torch
+
+
+def _dtype_code(t) -> int:
+    torch = _torch()
+    m = {torch.float32: KD_F32, torch.float16: KD_F16, torch.bfloat16: KD_BF16}
+    if t not in m:
+        raise TypeError(f"unsupported dtype {t}")
+    return m[t]
+
+
+def _ptr(t) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def _stream(stream) -> int:
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+class Workspace:
+    """Device scratch for one vector length (reusable across calls on one stream)."""
+
+    def __init__(self, n: int, device="cuda"):
+        torch = _torch()
+        self.n = int(n)
+        size = kd_workspace_size(self.n)
+        if size == 0:
+            raise KashinError(KD_ERR_UNSUPPORTED_N if kd_supported(self.n) else KD_ERR_CUDA,
+                              f"kd_workspace_size({self.n})")
+        self.nbytes = size
+        self.buf = torch.empty(size, dtype=torch.uint8, device=device)
+
+    @property
+    def ptr(self) -> int:
+        return self.buf.data_ptr()
+
+
+@dataclasses.dataclass
+class Decomposed:
+    codes_u: "object"     # int32 view of uint32 words, (m, ceil(n/16))
+    codes_v: "object"
+    centres_u: "object"   # float32 (m, 4)
+    centres_v: "object"
+    coeffs: "object"      # float32 (m, 4) or None
+    u: "object"           # float32 (m, n) or None
+    vhat: "object"
+    resid: "object"
+    trace: "object"       # int8 (m, 4*iters, n) or None
+
+
+def decompose(w, iters: int, sign_seed: int, layout: str = "rows", factors: bool = False,
+              coeffs: bool = True, trace: bool = False, workspace: Optional[Workspace] = None,
+              out: Optional[Decomposed] = None, stream=None) -> Decomposed:
+    """Decompose every vector of ``w`` (Alg. 1) and 2-bit code both factors.
+
+    ``layout='rows'``: ``w`` is (m, n), vector j = ``w[j]`` (nn.Linear weight).
+    ``layout='columns'``: ``w`` is (n, m), vector j = ``w[:, j]`` (the paper's W).
+    """
+    torch = _torch()
+    if not w.is_cuda:
+        raise ValueError("w must be a CUDA tensor")
+    if w.dim() != 2 or w.stride(1) != 1:
+        raise ValueError("w must be 2-D with unit inner stride")
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    if lay == KD_VEC_ROWS:
+        m, n = w.shape
+    else:
+        n, m = w.shape
+    ld = w.stride(0)
+    dev = w.device
+    words = (n + 15) // 16
+    if out is None:
+        f32 = dict(dtype=torch.float32, device=dev)
+        out = Decomposed(
+            codes_u=torch.empty((m, words), dtype=torch.int32, device=dev),
+            codes_v=torch.empty((m, words), dtype=torch.int32, device=dev),
+            centres_u=torch.empty((m, 4), **f32), centres_v=torch.empty((m, 4), **f32),
+            coeffs=torch.empty((m, 4), **f32) if coeffs else None,
+            u=torch.empty((m, n), **f32) if factors else None,
+            vhat=torch.empty((m, n), **f32) if factors else None,
+            resid=torch.empty((m, n), **f32) if factors else None,
+            trace=torch.empty((m, 4 * iters, n), dtype=torch.int8, device=dev) if trace else None)
+    ws = workspace if workspace is not None else Workspace(n, dev)
+    st = kd_decompose(w.data_ptr(), _dtype_code(w.dtype), lay, n, m, ld, sign_seed, int(iters),
+                      _ptr(out.codes_u), _ptr(out.codes_v), _ptr(out.centres_u), _ptr(out.centres_v),
+                      _ptr(out.coeffs), _ptr(out.u), _ptr(out.vhat), _ptr(out.resid), _ptr(out.trace),
+                      ws.ptr, ws.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_decompose")
+    return out
+
+
+def read_status(workspace: Workspace, stream=None) -> int:
+    return kd_read_status(workspace.ptr, _stream(stream))
+
+
+def apply_p(x, sign_seed: int, out=None, workspace: Optional[Workspace] = None, stream=None):
+    """``y_j = P x_j`` for the rows of the fp32 (m, n) tensor ``x``."""
+    torch = _torch()
+    if x.dtype != torch.float32 or not x.is_contiguous() or x.dim() != 2:
+        raise ValueError("x must be a contiguous fp32 (m, n) CUDA tensor")
+    m, n = x.shape
+    y = out if out is not None else torch.empty_like(x)
+    ws = workspace if workspace is not None else Workspace(n, x.device)
+    st = kd_apply_p(x.data_ptr(), y.data_ptr(), n, m, sign_seed, ws.ptr, ws.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_apply_p")
+    return y
+
+
+def reconstruct(dec: Decomposed, n: int, sign_seed: int, dtype=None, layout: str = "rows", out=None,
+                workspace: Optional[Workspace] = None, stream=None):
+    """Dense ``W_hat = U_q + P V_q`` from codes and centres (App. C)."""
+    torch = _torch()
+    dtype = dtype or torch.float32
+    m = dec.codes_u.shape[0]
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    dev = dec.codes_u.device
+    if out is None:
+        out = torch.empty((m, n) if lay == KD_VEC_ROWS else (n, m), dtype=dtype, device=dev)
+    ws = workspace if workspace is not None else Workspace(n, dev)
+    st = kd_reconstruct(dec.codes_u.data_ptr(), dec.codes_v.data_ptr(), dec.centres_u.data_ptr(),
+                        dec.centres_v.data_ptr(), n, m, sign_seed, _dtype_code(out.dtype), lay, out.data_ptr(),
+                        out.stride(0), ws.ptr, ws.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_reconstruct")
+    return out
+
+
+def unpack_codes(words, n: int):
+    """(m, ceil(n/16)) int32 words -> (m, n) int64 codes (host numpy)."""
+    w = np.asarray(words.cpu().numpy() if hasattr(words, "cpu") else words).astype(np.uint32).astype(np.uint64)
+    m = w.shape[0]
+    idx = np.arange(n)
+    return ((w[:, idx // 16] >> (2 * (idx % 16)).astype(np.uint64)) & np.uint64(3)).astype(np.int64).reshape(m, n)

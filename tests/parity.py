@@ -1,0 +1,133 @@
+"""Parity harness: compare device results with the CPU oracle on the same inputs.
+
+Tolerances (from the stated contract, per vector):
+  u, vhat      ||gpu - ora||_inf / ||ora||_inf <= 1e-5
+  coefficients |gpu - ora| / ora <= 1e-5 ; centres relative to their outer value
+  codes        identical, except entries whose oracle value lies within
+               1e-6 * (a1 + a2) of a decision boundary; those <= 0.01 % of entries
+  x = u + P vhat + r  from the device factors: relative l2 error <= 1e-6
+Signs: Alg. 1 takes sign() of every entry at every step; where fp32 and fp64
+disagree on a value within rounding of zero the trajectories would split, so
+the oracle follows the device's recorded sign wherever its own argument is
+within tau_abs = TAU * rms(x) of zero and counts any other disagreement as a
+hard failure (must be zero).
+"""
+
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+
+from oracle import kashin_oracle as ko
+
+TAU = 1e-5          # tie window, relative to the vector's rms
+TOL_FACTOR = 1e-5   # u, vhat, coefficients, centres
+TOL_RECON = 1e-6    # x = u + P vhat + r from device factors
+CODE_WINDOW = 1e-6  # near-boundary window, relative to a1 + a2
+CODE_FRAC = 1e-4    # at most 0.01 % of entries may differ, all inside the window
+
+
+@dataclasses.dataclass
+class ParityReport:
+    n: int
+    m: int
+    hard: int
+    ties: int
+    tie_flips: int
+    u_err: float
+    v_err: float
+    coef_err: float
+    cent_err: float
+    code_diff: int
+    code_diff_outside: int
+    code_near: int
+    recon_err: float
+    entries: int
+
+    def check(self):
+        assert self.hard == 0, f"{self.hard} sign decisions disagree outside the tie window"
+        assert self.u_err <= TOL_FACTOR, f"u max rel err {self.u_err:.3e}"
+        assert self.v_err <= TOL_FACTOR, f"vhat max rel err {self.v_err:.3e}"
+        assert self.coef_err <= TOL_FACTOR, f"coefficient rel err {self.coef_err:.3e}"
+        assert self.cent_err <= TOL_FACTOR, f"centre rel err {self.cent_err:.3e}"
+        assert self.code_diff_outside == 0, f"{self.code_diff_outside} code mismatches away from a boundary"
+        assert self.code_diff <= CODE_FRAC * self.entries, f"{self.code_diff} code mismatches"
+        assert self.recon_err <= TOL_RECON, f"x = u + P vhat + r rel err {self.recon_err:.3e}"
+
+
+def _rel_inf(a, b):
+    """max over columns of ||a-b||_inf / ||b||_inf (columns with b == 0 use abs error)."""
+    num = np.abs(a - b).max(axis=0)
+    den = np.abs(b).max(axis=0)
+    out = np.where(den > 0, num / np.where(den > 0, den, 1), num)
+    return float(out.max()) if out.size else 0.0
+
+
+def compare(x: np.ndarray, seed: int, iters: int, dev: dict, P_oracle=None) -> ParityReport:
+    """x: (N, M) float64 inputs (exact values the device saw).  dev: numpy arrays
+    from the device, vector-major: u, vhat, resid (M, N) float32, coeffs (M, 4),
+    centres_u/centres_v (M, 4), codes_u/codes_v (M, N) int, trace (M, 4k, N) int8."""
+    N, M = x.shape
+    eps = ko.sign_mask(seed, N)
+    P = P_oracle if P_oracle is not None else ko.POperator(N, eps)
+    rms = np.sqrt((x ** 2).mean(axis=0))
+    follow = np.transpose(dev["trace"], (1, 2, 0)).astype(np.int8)   # (4k, N, M)
+    d = ko.decompose(x, eps, iters, follow=follow, tau_abs=TAU * rms, P=P)
+    cu = ko.centres(d.coeffs[0], d.coeffs[1])
+    cv = ko.centres(d.coeffs[2], d.coeffs[3])
+    code_u = ko.codes(d.u, cu)
+    code_v = ko.codes(d.vhat, cv)
+
+    u_g = dev["u"].T.astype(np.float64)
+    v_g = dev["vhat"].T.astype(np.float64)
+    r_g = dev["resid"].T.astype(np.float64)
+    u_err = _rel_inf(u_g, d.u)
+    v_err = _rel_inf(v_g, d.vhat)
+    co_g = dev["coeffs"].T.astype(np.float64)
+    den = np.where(d.coeffs != 0, np.abs(d.coeffs), 1.0)
+    coef_err = float((np.abs(co_g - d.coeffs) / den).max()) if M else 0.0
+    cent_err = 0.0
+    for cg, co in ((dev["centres_u"], cu), (dev["centres_v"], cv)):
+        outer = np.abs(co[:, 3])
+        dd = np.abs(cg.astype(np.float64) - co).max(axis=1)
+        cent_err = max(cent_err, float(np.where(outer > 0, dd / np.where(outer > 0, outer, 1), dd).max()))
+
+    diff = 0
+    outside = 0
+    near_total = 0
+    for cg, co, vals, cent in ((dev["codes_u"], code_u, d.u, cu), (dev["codes_v"], code_v, d.vhat, cv)):
+        cg = cg.T
+        mism = cg != co
+        dist = ko.boundary_distance(vals, cent)
+        window = CODE_WINDOW * np.abs(cent[:, 3])[None, :]
+        near = dist <= window
+        near_total += int(near.sum())
+        diff += int(mism.sum())
+        outside += int((mism & ~near).sum())
+
+    Pv = P(v_g)
+    recon = np.linalg.norm(x - u_g - Pv - r_g, axis=0) / np.where(np.linalg.norm(x, axis=0) > 0,
+                                                                  np.linalg.norm(x, axis=0), 1)
+    return ParityReport(n=N, m=M, hard=d.hard_mismatches, ties=d.ties, tie_flips=d.tie_flips, u_err=u_err,
+                        v_err=v_err, coef_err=coef_err, cent_err=cent_err, code_diff=diff,
+                        code_diff_outside=outside, code_near=near_total, recon_err=float(recon.max()),
+                        entries=2 * N * M)
+
+
+def device_outputs(kd, w_dev, iters, seed, trace=True, layout="rows"):
+    """Run kd_decompose with every optional output and return numpy arrays."""
+    out = kd.decompose(w_dev, iters, seed, layout=layout, factors=True, coeffs=True, trace=trace)
+    n = out.u.shape[1]
+    import torch
+    torch.cuda.synchronize()
+    res = {
+        "u": out.u.cpu().numpy(), "vhat": out.vhat.cpu().numpy(), "resid": out.resid.cpu().numpy(),
+        "coeffs": out.coeffs.cpu().numpy(), "centres_u": out.centres_u.cpu().numpy(),
+        "centres_v": out.centres_v.cpu().numpy(),
+        "codes_u": kd.unpack_codes(out.codes_u, n), "codes_v": kd.unpack_codes(out.codes_v, n),
+        "words_u": out.codes_u.cpu().numpy(), "words_v": out.codes_v.cpu().numpy(),
+    }
+    if trace:
+        res["trace"] = out.trace.cpu().numpy()
+    return res

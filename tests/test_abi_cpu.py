@@ -1,0 +1,112 @@
+"""C-ABI checks that need no GPU: the library builds/loads, exports every entry
+point include/kashin.h declares, and its host-only logic (sign mask, plan
+lookup, workspace sizing, argument validation) behaves.  No kernel is launched."""
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+from oracle import kashin_oracle as ko
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "kashin.h")
+
+
+@pytest.fixture(scope="module")
+def kd():
+    from paper_2609_11687_gb300 import build
+    build.build()
+    from paper_2609_11687_gb300 import kashin
+    return kashin
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(kd_[a-z_]+)\s*\(", src)))
+
+
+def test_header_declares_expected_entry_points():
+    names = declared_functions()
+    for must in ("kd_decompose", "kd_reconstruct", "kd_apply_p", "kd_signs", "kd_workspace_size",
+                 "kd_read_status", "kd_supported", "kd_status_string", "kd_version"):
+        assert must in names
+
+
+def test_library_exports_every_declared_symbol(kd):
+    lib = ctypes.CDLL(kd.LIB_PATH)
+    for name in declared_functions():
+        assert hasattr(lib, name), f"{name} declared in kashin.h but not exported"
+    assert set(declared_functions()) <= set(kd.EXPORTS)
+
+
+def test_version_and_status_strings(kd):
+    assert "libkashin" in kd.version()
+    assert kd.status_string(kd.KD_OK) == "KD_OK"
+    assert kd.status_string(kd.KD_ERR_NONFINITE) == "KD_ERR_NONFINITE"
+    assert kd.status_string(99) == "KD_ERR_UNKNOWN"
+
+
+@pytest.mark.parametrize("seed,n", [(0, 16), (1, 257), (0xDEADBEEFCAFEF00D, 4096), (2**64 - 1, 100)])
+def test_kd_signs_match_oracle(kd, seed, n):
+    np.testing.assert_array_equal(kd.kd_signs(seed, n), ko.sign_mask(seed, n).astype(np.int8))
+
+
+def test_supported_lengths(kd):
+    for n in (16, 256, 768, 3072, 4096, 11008, 14336, 16384):
+        assert kd.kd_supported(n) == kd.KD_OK
+    for n in (0, 1, 15, 100, 4095, 32768):
+        assert kd.kd_supported(n) == kd.KD_ERR_UNSUPPORTED_N
+
+
+def test_workspace_size_register_plans(kd):
+    # plans that keep u in registers need only the tables: no device query
+    for n in (256, 768, 4096):
+        ws = kd.kd_workspace_size(n)
+        assert ws >= 256 + 16 * n and ws % 256 == 0
+    assert kd.kd_workspace_size(100) == 0
+
+
+def test_argument_validation_without_gpu(kd):
+    null = None
+    # unsupported length
+    st = kd.kd_decompose(1, 0, 0, 100, 4, 100, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20, null)
+    assert st == kd.KD_ERR_UNSUPPORTED_N
+    # negative iterations / bad dtype / bad layout / ld too small
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, -1, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose(1, 7, 0, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose(1, 0, 5, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 255, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    # missing required outputs
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, null, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    # workspace missing / too small
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, null, 1 << 20,
+                           null) == kd.KD_ERR_WORKSPACE
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 16,
+                           null) == kd.KD_ERR_WORKSPACE
+    assert kd.kd_apply_p(1, 1, 256, 2, 0, null, 0, null) == kd.KD_ERR_WORKSPACE
+    assert kd.kd_apply_p(null, 1, 256, 2, 0, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_reconstruct(1, 1, 1, 1, 256, 2, 0, 9, 0, 1, 256, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_read_status(null, null) == kd.KD_ERR_WORKSPACE
+
+
+def test_product_path_requires_library(tmp_path, monkeypatch):
+    """Importing the binding without the built library raises: no CPU fallback."""
+    import importlib.util
+    import shutil
+    pkg = tmp_path / "pkgcopy"
+    pkg.mkdir()
+    src = os.path.join(ROOT, "paper_2609_11687_gb300", "kashin.py")
+    shutil.copy(src, pkg / "kashin.py")
+    spec = importlib.util.spec_from_file_location("kashin_nolib", pkg / "kashin.py")
+    mod = importlib.util.module_from_spec(spec)
+    with pytest.raises(ImportError):
+        spec.loader.exec_module(mod)
