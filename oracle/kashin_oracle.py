@@ -127,7 +127,8 @@ def _sign(a: np.ndarray) -> np.ndarray:
 
 
 def decompose(x: np.ndarray, eps: np.ndarray, iters: int, follow: Optional[np.ndarray] = None,
-              tau_abs: Optional[np.ndarray] = None, P: Optional[POperator] = None) -> Decomposition:
+              tau_abs: Optional[np.ndarray] = None, P: Optional[POperator] = None,
+              follow_floor: Optional[np.ndarray] = None) -> Decomposition:
     """Run Algorithm 1 on every column of ``x`` (shape ``(N, M)``), float64.
 
     Per block t (k blocks): two greedy steps on the cube vertices Q_N update u,
@@ -140,7 +141,12 @@ def decompose(x: np.ndarray, eps: np.ndarray, iters: int, follow: Optional[np.nd
     given (int8, shape ``(4k, N, M)``: the sign the device took at every atomic
     step, in natural element order), then wherever the oracle's own argument has
     ``|arg| <= tau_abs[col]`` the followed sign is used instead; a disagreement
-    where ``|arg| > tau_abs`` is counted in ``hard_mismatches``.
+    where ``|arg| > tau_abs`` is counted in ``hard_mismatches``.  Following only
+    happens while the step's residual norm ``||rho||_2`` is at least
+    ``follow_floor[col]`` (the device's rounding floor): below it the device's
+    signs are rounding noise, so the oracle takes its own and counts nothing;
+    each such step moves u or vhat by at most ``||rho||_2 / sqrt(N)``
+    (Eq. lambda_bound).
     """
     x = np.asarray(x, dtype=np.float64)
     if x.ndim == 1:
@@ -162,6 +168,10 @@ def decompose(x: np.ndarray, eps: np.ndarray, iters: int, follow: Optional[np.nd
             return own
         dev = follow[step].astype(np.float64)
         near = np.abs(arg) <= tau_abs[None, :]
+        if follow_floor is not None:
+            resolved = np.linalg.norm(arg, axis=0) >= follow_floor
+            dev = np.where(resolved[None, :], dev, own)
+            near = near & resolved[None, :]
         stats["ties"] += int(near.sum())
         stats["flips"] += int((near & (dev != own)).sum())
         stats["hard"] += int((~near & (dev != own)).sum())

@@ -1,21 +1,17 @@
 // Launch helpers shared by the per-N translation units.
 #pragma once
-#include <mutex>
 
 #include "kd_kernels.cuh"
 #include "kd_ops.h"
 
 namespace kd {
 
+// Opt the kernel in to its dynamic shared memory (> 48 KB for large N).  Done on
+// every launch: the attribute is per function and per device, and the call
+// costs about a microsecond next to millisecond-scale kernels.
 template <class K>
 inline cudaError_t prepare(K kernel, size_t smem) {
-  // Opt in to more than 48 KB of dynamic shared memory, once per kernel.
-  static std::once_flag once;
-  static cudaError_t err = cudaSuccess;
-  std::call_once(once, [&] {
-    err = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  });
-  return err;
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
 }
 
 template <class K>

@@ -314,3 +314,17 @@ def test_reconstruct_n2():
     W = ko.reconstruct(code_u, code_v, cu, cv, eps)
     # U_q = (2, -2); V_q = (-3, 3); P = swap -> P V_q = (3, -3)
     np.testing.assert_allclose(W[:, 0], [5.0, -5.0], atol=1e-14)
+
+
+def test_follow_floor_gates_following():
+    """Below the follow floor the oracle takes its own signs and counts nothing."""
+    N, k = 64, 3
+    x = _gauss(N, 2, seed=6)
+    eps = ko.sign_mask(6, N)
+    ref = ko.decompose(x, eps, k)
+    planted = np.zeros((4 * k, N, 2), dtype=np.int8)          # a device that always says 0
+    gated = ko.decompose(x, eps, k, follow=planted, tau_abs=np.full(2, 1e9), follow_floor=np.full(2, 1e9))
+    assert gated.ties == 0 and gated.hard_mismatches == 0
+    np.testing.assert_array_equal(gated.u, ref.u)
+    open_gate = ko.decompose(x, eps, k, follow=planted, tau_abs=np.full(2, 1e9), follow_floor=np.zeros(2))
+    assert open_gate.ties == 4 * k * N * 2
