@@ -1,0 +1,424 @@
+"""Benchmark: parameters decomposed + 2-bit coded per second at Llama-2-7B layer shapes.
+
+One step = Algorithm 1 (k blocks) + closed-form centres + packed 2-bit codes for every
+vector of one Llama-2-7B-shaped decoder layer (q, k, v, o: 4096x4096; gate, up:
+4096x11008; down: 11008x4096 -- 202,375,168 parameters), through the C ABI
+(kd_decompose, one call per matrix).  Steps cycle through the 32 layers of the
+seeded 7B-shaped stack, generated once on the device and resident in HBM (13 GB
+fp16), so no step re-reads an input another step touched; every input is larger
+than L2.
+
+Prints ONE JSON line on rank 0.  Extras in that line:
+  roofline      ALU roofline of the dominant kernel (decompose, N = 4096), measured
+                with CUDA events on the launch stream inside the timed region.
+  cpu_baseline  the CPU oracle (fp64, dense DCT matrix) on a bounded sample.
+  e2e           same metric with host (pinned) input buffers, H2D + D2H in the loop.
+  clocks        nvidia-smi samples taken during the timed region.
+
+``--impl reference`` times the CPU oracle instead (the reference arm).
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "params decomposed+2-bit coded/sec at 7B layer shapes; % of roofline"
+UNIT = "params/s"
+ITERS = 16
+LAYERS = 32
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+PROFILE_FILE = os.path.join(ROOT, "profiles", "decompose_n4096_llama7b.json")
+SM_COUNT = 152
+FP32_LANES_PER_SM = 128
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def flops_per_vector(n: int, iters: int) -> float:
+    """Algorithmic FP32 work of Algorithm 1 on one vector (fixed convention):
+    per block 4 length-n DCTs at 2 n log2 n each + 20 n for the four greedy steps."""
+    return iters * (4 * 2 * n * math.log2(n) + 20 * n)
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_11687_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-f", self.path], stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = sorted(float(r[1]) for r in rows if r[1].replace(".", "").isdigit())
+        mx = max(float(r[2]) for r in rows if r[2].replace(".", "").isdigit())
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        power = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        return {"sm_mhz": sm[len(sm) // 2] if sm else None, "sm_max_mhz": mx, "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(power) if power else None}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle baseline (bounded sample)
+# ---------------------------------------------------------------------------
+
+def oracle_baseline(specs, iters: int, budget_s: float = 12.0) -> dict:
+    """Time the CPU oracle as it stands on a bounded sample of the layer and scale
+    to params/s of the whole layer mix (time per parameter measured per vector
+    length, weighted by the layer's parameters at that length)."""
+    import numpy as np
+    from oracle import kashin_oracle as ko
+    from paper_2609_11687_gb300 import synth
+    by_n = {}
+    for s in specs:
+        by_n.setdefault(s.N, []).append(s)
+    per_param = {}
+    sample_desc = []
+    share = budget_s / len(by_n)
+    for n, group in sorted(by_n.items()):
+        spec = group[0]
+        import torch
+        import dataclasses
+        G = synth.generate(dataclasses.replace(spec, M=64))
+        x = G.double().numpy().T
+        eps = ko.sign_mask(spec.sign_seed, n)
+        P = ko.POperator(n, eps)
+        m = 2
+        while True:
+            t0 = time.perf_counter()
+            ko.decompose(x[:, :m], eps, iters, P=P)
+            dt = time.perf_counter() - t0
+            if dt > share / 4 or m >= 64:
+                break
+            m = min(64, m * 2)
+        per_param[n] = dt / (m * n)
+        sample_desc.append(f"{m} vectors of n={n} ({dt:.1f}s)")
+    layer_params = sum(s.params for s in specs)
+    layer_time = sum(s.params * per_param[s.N] for s in specs)
+    return {"value": layer_params / layer_time, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+            "sample": "fp64 dense-DCT oracle, k=%d, on %s, scaled to the layer's parameter mix (seeded "
+                      "Student-t vectors of the layer's shapes)" % (iters, "; ".join(sample_desc))}
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_gpu(args) -> dict:
+    import torch
+    from paper_2609_11687_gb300 import build, synth
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    build.build()
+    from paper_2609_11687_gb300 import kashin as kd
+
+    iters = args.iters
+    dev = torch.device("cuda", local)
+    # this rank's layers: rank, rank + world, ...  (weak scaling, no data exchange)
+    steps_total = args.warmup + args.steps
+    my_layers = [(rank + world * i) % LAYERS for i in range(steps_total)]
+    uniq = sorted(set(my_layers))
+    log(f"[bench] rank {rank}/{world}: generating {len(uniq)} Llama-2-7B-shaped layers on {dev}")
+    t0 = time.time()
+    layers = {}
+    for L in uniq:
+        specs = synth.llama7b_layer(L)
+        layers[L] = [(s, synth.generate(s, device=dev)) for s in specs]
+    torch.cuda.synchronize()
+    log(f"[bench] generated in {time.time() - t0:.1f}s")
+    layer_params = synth.total_params(synth.llama7b_layer(0))
+
+    # outputs and workspaces, allocated once
+    outs = {}
+    wss = {}
+    for s, w in layers[uniq[0]]:
+        key = (s.N, s.M)
+        if key not in outs:
+            words = (s.N + 15) // 16
+            outs[key] = kd.Decomposed(
+                codes_u=torch.empty((s.M, words), dtype=torch.int32, device=dev),
+                codes_v=torch.empty((s.M, words), dtype=torch.int32, device=dev),
+                centres_u=torch.empty((s.M, 4), dtype=torch.float32, device=dev),
+                centres_v=torch.empty((s.M, 4), dtype=torch.float32, device=dev),
+                coeffs=None, u=None, vhat=None, resid=None, trace=None)
+        if s.N not in wss:
+            wss[s.N] = kd.Workspace(s.N, dev)
+    stream = torch.cuda.current_stream()
+
+    ev_main = {}  # per-launch events of the dominant kernel (N = 4096)
+
+    def run_layer(L, record=False):
+        for s, w in layers[L]:
+            o = outs[(s.N, s.M)]
+            if record and s.N == 4096:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream)
+            if record and s.N == 4096:
+                e1.record(stream)
+                ev_main.setdefault("ev", []).append((e0, e1, s.M))
+
+    for i in range(args.warmup):
+        run_layer(my_layers[i])
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    start.record(stream)
+    for i in range(args.steps):
+        run_layer(my_layers[args.warmup + i], record=True)
+    end.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    clk = clocks.stop()
+    elapsed_ms = start.elapsed_time(end)
+    t = torch.tensor([elapsed_ms], device=dev)
+    if dist:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    elapsed_ms = float(t.item())
+    value = world * args.steps * layer_params / (elapsed_ms / 1e3)
+
+    # dominant kernel: average launch duration over the timed region
+    launches = ev_main.get("ev", [])
+    dur = sum(a.elapsed_time(b) for a, b, _ in launches) / max(1, len(launches))
+    vec_per_launch = sum(mm for _, _, mm in launches) / max(1, len(launches))
+    fl = flops_per_vector(4096, iters) * vec_per_launch
+    achieved_tflops = fl / (dur / 1e3) / 1e12
+    peak = SM_COUNT * FP32_LANES_PER_SM * 2 * 2.070e9 / 1e12
+    traffic = None
+    if os.path.exists(PROFILE_FILE):
+        with open(PROFILE_FILE) as f:
+            prof = json.load(f)
+        if prof.get("kernel_hash") == kernel_source_hash() and prof.get("iters") == iters:
+            traffic = prof["dram_bytes_per_vector"] * vec_per_launch
+    roofline = {"bound": "alu", "achieved": round(achieved_tflops, 3), "peak": round(peak, 2),
+                "unit": "TFLOP/s", "frac": round(achieved_tflops / peak, 4), "traffic": traffic,
+                "kernel": "decompose_kernel<N=4096>", "launch_ms": round(dur, 3),
+                "peak_basis": "FP32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz (max clock)"}
+    if clk.get("sm_mhz"):
+        roofline["frac_at_measured_clock"] = round(achieved_tflops / (peak * clk["sm_mhz"] / 2070.0), 4)
+
+    # end to end: pinned host input, H2D + decompose + D2H codes/centres each step
+    e2e = None
+    if not args.skip_e2e:
+        e2e = run_e2e(kd, torch, layers[uniq[0]], outs, wss, iters, args, stream, dist, world)
+
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "llama2-7b decoder layer per step: q,k,v,o 4096x4096, gate,up 4096x11008, "
+                               "down 11008x4096 (202,375,168 params, fp16 Student-t nu=4 std 0.015, 0.1% input "
+                               "channels x20), cycling the 32 seeded layers of the 7B stack resident in HBM",
+                   "iters": iters, "layout": "vector-major (nn.Linear [out, in])",
+                   "l2": "inputs larger than L2 (405 MB per step, distinct layer every step)",
+                   "parallelism": f"dp{world} (layers sharded over ranks, no exchange)"},
+        "roofline": roofline,
+        "gpu_launches": args.steps * 7 * 2,
+        "clocks": clk,
+    }
+    if e2e is not None:
+        result["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.skip_cpu:
+        result["cpu_baseline"] = oracle_baseline(synth.llama7b_layer(0), iters, budget_s=args.cpu_budget)
+    if dist:
+        dist.destroy_process_group()
+    return result if rank == 0 else None
+
+
+def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
+    """Same metric through the C ABI with host buffers: every step copies the
+    layer's fp16 weights from pinned host memory and reads codes + centres back."""
+    host_in = [(s, w.cpu().pin_memory()) for s, w in layer]
+    dev_in = [torch.empty_like(w, device=stream.device) for _, w in layer]
+    host_out = {k: (torch.empty(o.codes_u.shape, dtype=torch.int32).pin_memory(),
+                    torch.empty(o.codes_v.shape, dtype=torch.int32).pin_memory(),
+                    torch.empty(o.centres_u.shape).pin_memory(), torch.empty(o.centres_v.shape).pin_memory())
+                for k, o in outs.items()}
+    h2d = sum(w.numel() * w.element_size() for _, w in host_in)
+    d2h = 0
+    for s, _ in layer:
+        o = outs[(s.N, s.M)]
+        d2h += sum(t.numel() * t.element_size() for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v))
+
+    def step():
+        for (s, hw), dw in zip(host_in, dev_in):
+            dw.copy_(hw, non_blocking=True)
+            o = outs[(s.N, s.M)]
+            kd.decompose(dw, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream)
+            hu, hv, hcu, hcv = host_out[(s.N, s.M)]
+            hu.copy_(o.codes_u, non_blocking=True)
+            hv.copy_(o.codes_v, non_blocking=True)
+            hcu.copy_(o.centres_u, non_blocking=True)
+            hcv.copy_(o.centres_v, non_blocking=True)
+
+    for _ in range(2):
+        step()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    n = max(1, args.steps // 4)
+    a.record(stream)
+    for _ in range(n):
+        step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b)
+    t = torch.tensor([ms], device=stream.device)
+    if dist:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms = float(t.item())
+    params = sum(s.params for s, _ in layer)
+    return {"value": round(world * n * params / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": d2h, "steps": n}
+
+
+# ---------------------------------------------------------------------------
+# reference arm: the CPU oracle as it stands
+# ---------------------------------------------------------------------------
+
+def run_reference(args) -> dict | None:
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return None
+    from paper_2609_11687_gb300 import synth
+    specs = synth.llama7b_layer(0)
+    budget = max(2.0, min(30.0, 150.0 / max(1, args.steps + args.warmup)))
+    vals = []
+    for i in range(args.warmup + args.steps):
+        b = oracle_baseline(specs, args.iters, budget_s=budget)
+        if i >= args.warmup:
+            vals.append(b)
+    value = sum(v["value"] for v in vals) / len(vals)
+    layer_params = synth.total_params(specs)
+    return {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": layer_params / value * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "llama2-7b decoder layer per step (202,375,168 params), each timed step a "
+                               "bounded sample of that layer on the host cores", "iters": args.iters},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": vals[-1]["sample"]},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+
+
+def run_profile_case(args) -> None:
+    """Small case for ncu: one 4096 x M fp16 matrix of the layer's distribution
+    (M = 32768 vectors: 256 MB of input, above L2), decomposed 3 times."""
+    import dataclasses
+    import torch
+    from paper_2609_11687_gb300 import build, synth
+    build.build()
+    from paper_2609_11687_gb300 import kashin as kd
+    spec = dataclasses.replace(synth.llama7b_layer(0)[0], M=args.profile_m)
+    w = synth.generate(spec, device="cuda")
+    ws = kd.Workspace(spec.N)
+    out = None
+    for _ in range(3):
+        out = kd.decompose(w, args.iters, spec.sign_seed, workspace=ws, out=out)
+    torch.cuda.synchronize()
+    log(f"[profile-case] ok: n={spec.N} m={spec.M} iters={args.iters}")
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=32)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--iters", type=int, default=ITERS)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--skip-cpu", action="store_true")
+    ap.add_argument("--skip-e2e", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
+    ap.add_argument("--profile-m", type=int, default=32768)
+    args = ap.parse_args()
+    if args.profile_case:
+        run_profile_case(args)
+        return
+    if args.warmup < 3:
+        log("[bench] warmup raised to 3 (timing rule)")
+        args.warmup = 3
+    res = run_reference(args) if args.impl == "reference" else run_gpu(args)
+    if res is not None:
+        print(json.dumps(res), flush=True)
+
+
+if __name__ == "__main__":
+    main()

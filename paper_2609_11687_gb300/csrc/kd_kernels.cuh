@@ -356,6 +356,15 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
       if (finB && cB > 0.f) sB = max(-100, min(100, -ilogbf(cB)));
     }
     const float scA = pow2f(sA), scB = pow2f(sB);
+    // An all-zero vector must stay exactly zero; the packed transform would
+    // otherwise leak its partner's rounding error into it.
+    const bool liveA = sum0.x > 0.f, liveB = sum0.y > 0.f;
+    auto mask_dead = [&](float2(&v)[E]) {
+      if (!liveA || !liveB) {
+#pragma unroll
+        for (int j = 0; j < E; ++j) v[j] = make_float2(liveA ? v[j].x : 0.f, liveB ? v[j].y : 0.f);
+      }
+    };
 #pragma unroll
     for (int j = 0; j < E; ++j) r[j] = make_float2(__fmul_rn(r[j].x, scA), __fmul_rn(r[j].y, scB));
     sum0 = make_float2(__fmul_rn(sum0.x, scA), __fmul_rn(sum0.y, scB));
@@ -444,11 +453,13 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
       }
       // two greedy steps from P Q_N on y = P rho (update vhat implicitly)
       apply_P<PL>(r, buf, p.tw, p.eps, lt);
+      mask_dead(r);
       float2 l3 = greedy(step, false, sum0, add_none);
       ++step;
       float2 l4 = greedy(step, false, sum0, add_none);
       ++step;
       apply_P<PL>(r, buf, p.tw, p.eps, lt);
+      mask_dead(r);
       if (t == 0) {
         coef[0] = l1;
         coef[1] = l2;
@@ -474,6 +485,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
     }
     if (p.iters > 0) {
       apply_P<PL>(vh, buf, p.tw, p.eps, lt);
+      mask_dead(vh);
     } else {
 #pragma unroll
       for (int j = 0; j < E; ++j) vh[j] = make_float2(0.f, 0.f);

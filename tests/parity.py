@@ -50,14 +50,18 @@ class ParityReport:
     recon_err: float
     entries: int
 
-    def check(self):
+    def check(self, code_budget: bool = True):
+        """code_budget=False for degenerate inputs (constant vectors, single spikes)
+        whose values sit on a decision boundary by construction: every mismatch
+        must still lie inside the boundary window."""
         assert self.hard == 0, f"{self.hard} sign decisions disagree outside the tie window"
         assert self.u_err <= TOL_FACTOR, f"u max rel err {self.u_err:.3e}"
         assert self.v_err <= TOL_FACTOR, f"vhat max rel err {self.v_err:.3e}"
         assert self.coef_err <= TOL_FACTOR, f"coefficient rel err {self.coef_err:.3e}"
         assert self.cent_err <= TOL_FACTOR, f"centre rel err {self.cent_err:.3e}"
         assert self.code_diff_outside == 0, f"{self.code_diff_outside} code mismatches away from a boundary"
-        assert self.code_diff <= CODE_FRAC * self.entries, f"{self.code_diff} code mismatches"
+        if code_budget:
+            assert self.code_diff <= CODE_FRAC * self.entries, f"{self.code_diff} code mismatches"
         assert self.recon_err <= TOL_RECON, f"x = u + P vhat + r rel err {self.recon_err:.3e}"
 
 

@@ -126,7 +126,7 @@ def test_zero_and_sparse_vectors(kd, torch_mod):
     G[3, 17] = 0.5                       # a single spike
     G[4] = 1e-3                          # constant vector
     rep, dev = _parity(kd, torch, G, seed=5)
-    rep.check()
+    rep.check(code_budget=False)   # the constant and spike vectors sit on boundaries by construction
     assert not dev["u"][1].any() and not dev["vhat"][1].any()
     assert not dev["centres_u"][1].any()
     assert not dev["words_u"][1].any()
