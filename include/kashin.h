@@ -108,6 +108,26 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
                        float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
                        void* workspace, size_t ws_bytes, void* stream);
 
+/* kd_decompose without a caller workspace, for callers that cannot allocate device
+ * memory (a plugin whose host application owns every device allocation and forbids
+ * direct cudaMalloc, or a loop that cannot afford cudaMalloc's implicit
+ * synchronisation).  The paper has no counterpart: this is a library convenience.
+ * Same arguments and results as kd_decompose minus workspace/ws_bytes; the scratch
+ * lives in a 160 KB static device array inside the library instead.
+ *   - n <= 8192 only; larger n returns KD_ERR_WORKSPACE and enqueues nothing.
+ *   - Allocates nothing.  Every GPU that loads the library holds the array until exit.
+ *   - All calls share the array (it keeps the last call's tables); each call rewrites
+ *     what it needs on its own stream, so calls that overlap on the GPU race.
+ *   - The first call on a device resolves the array's address (cudaGetSymbolAddress,
+ *     once per device): make that first call before any stream capture.
+ *   - Non-finite inputs still set the device status word, which lives in the static
+ *     array and is not readable through this ABI. */
+kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
+                              int64_t ld, uint64_t sign_seed, int iters,
+                              uint32_t* codes_u, uint32_t* codes_v, float* centres_u, float* centres_v,
+                              float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
+                              void* stream);
+
 /* y_j = P x_j for m vectors of length n, fp32, vector-major [m][n] contiguous
  * (Sec. 3.1: P z = IDCT(eps * DCT(z)); App. C uses the same operator on the rows
  * of the activations, XP).  x and y may alias. */

@@ -30,7 +30,7 @@ KD_F32, KD_F16, KD_BF16 = 0, 1, 2
 KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
-           "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status")
+           "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static")
 
 
 def _load() -> ctypes.CDLL:
