@@ -1,0 +1,62 @@
+"""Full-size parity: every matrix of the 7B-shaped workloads is decomposed whole,
+in the launch configuration bench.py times (one kd_decompose per matrix, inputs
+generated on the device); sampled vector pairs are then re-run with the trace on
+a gathered copy (pairs kept whole, so the arithmetic is identical) and checked
+
+  * bitwise against the full-size run (codes, centres, coefficients), and
+  * against the CPU oracle with the tie-following protocol of tests/parity.py.
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+
+from paper_2609_11687_gb300 import synth
+from tests import parity
+
+pytestmark = pytest.mark.gpu
+
+ITERS = 16
+SAMPLE_VECTORS = 32   # 16 pairs per matrix
+
+
+def _cases():
+    out = [("cfg3", s) for s in synth.config3()]
+    out += [("cfg4", s) for s in synth.config4(layers=[31])]
+    c5 = synth.config5(layers=[0, 31])
+    out += [("cfg5", s) for s in c5 if s.name.startswith("pythia.L31") or s.name.startswith("mistral.L0")]
+    return out
+
+
+CASES = _cases()
+
+
+@pytest.fixture(scope="module")
+def kd():
+    import torch
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2609_11687_gb300 import build
+    build.build()
+    from paper_2609_11687_gb300 import kashin
+    return kashin
+
+
+@pytest.mark.parametrize("cfg,spec", CASES, ids=[f"{c}-{s.name}" for c, s in CASES])
+def test_fullsize_sampled_parity(kd, cfg, spec):
+    import torch
+    w = synth.generate(spec, device="cuda")                  # (M, N) fp16, device generator
+    full = kd.decompose(w, ITERS, spec.sign_seed, coeffs=True)
+    idx = synth.pair_aligned_sample(spec.M, SAMPLE_VECTORS, seed=spec.seed + 17)
+    sub = w[idx].contiguous()
+    dev = parity.device_outputs(kd, sub, ITERS, spec.sign_seed, trace=True)
+    torch.cuda.synchronize()
+    sel = torch.tensor(idx, device="cuda")
+    for name in ("centres_u", "centres_v", "coeffs"):
+        np.testing.assert_array_equal(getattr(full, name)[sel].cpu().numpy(), dev[name], err_msg=name)
+    np.testing.assert_array_equal(full.codes_u[sel].cpu().numpy(), dev["words_u"])
+    np.testing.assert_array_equal(full.codes_v[sel].cpu().numpy(), dev["words_v"])
+    x = sub.double().cpu().numpy().T
+    rep = parity.compare(x, spec.sign_seed, ITERS, dev)
+    print(cfg, spec.name, rep)
+    rep.check()
