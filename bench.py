@@ -379,14 +379,14 @@ def run_reference(args) -> dict | None:
 
 
 def run_profile_case(args) -> None:
-    """Small case for ncu: one 4096 x M fp16 matrix of the layer's distribution
-    (M = 32768 vectors: 256 MB of input, above L2), decomposed 3 times."""
+    """Small case for ncu: one matrix of the layer's distribution with M vectors
+    (default q: n = 4096, M = 32768, 256 MB of input, above L2), decomposed 3 times."""
     import dataclasses
     import torch
     from paper_2609_11687_gb300 import build, synth
     build.build()
     from paper_2609_11687_gb300 import kashin as kd
-    spec = dataclasses.replace(synth.llama7b_layer(0)[0], M=args.profile_m)
+    spec = dataclasses.replace(synth.llama7b_layer(0)[args.profile_matrix], M=args.profile_m)
     w = synth.generate(spec, device="cuda")
     ws = kd.Workspace(spec.N)
     out = None
@@ -408,6 +408,7 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
     ap.add_argument("--profile-m", type=int, default=32768)
+    ap.add_argument("--profile-matrix", type=int, default=0, help="layer matrix index (0 = q, 6 = down)")
     args = ap.parse_args()
     if args.profile_case:
         run_profile_case(args)

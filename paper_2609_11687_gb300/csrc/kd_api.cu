@@ -37,45 +37,12 @@ const PlanOps* plan_ops(int64_t n) {
 
 namespace {
 
-// ---------------------------------------------------------------------------
-// Per-call tables: twiddles W_{2N}^j (double-precision sincospi, rounded) and the
-// sign mask bits (SplitMix64 of seed + (j+1)*gamma, bit 63 set -> eps_j = -1).
-// ---------------------------------------------------------------------------
-__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-
-__global__ void setup_tables_kernel(float2* tw, uint32_t* eps, uint32_t* status, int n, uint64_t seed) {
-  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
-  const int stride = gridDim.x * blockDim.x;
-  if (tid == 0) *status = 0u;
-  for (int j = tid; j < 2 * n; j += stride) {
-    double s, c;
-    sincospi((double)j / (double)n, &s, &c);
-    tw[j] = make_float2((float)c, (float)(-s));
-  }
-  const int words = (n + 31) / 32;
-  for (int wd = tid; wd < words; wd += stride) {
-    uint32_t bits = 0;
-    for (int b = 0; b < 32; ++b) {
-      const int j = wd * 32 + b;
-      if (j >= n) break;
-      const uint64_t z = splitmix64_mix(seed + (uint64_t)(j + 1) * 0x9E3779B97F4A7C15ull);
-      bits |= (uint32_t)(z >> 63) << b;
-    }
-    eps[wd] = bits;
-  }
-}
-
-
 constexpr size_t kAlign = 256;
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
-// Workspace layout: [status word | pad][twiddles 2n float2][sign bits][u slots]
+// Workspace layout: [status word | pad][sign bits][access-ordered twiddles][u slots]
 struct WsLayout {
-  size_t status, tw, eps, uslots, total;
+  size_t status, eps, tw, uslots, total;
 };
 
 int sm_count() {
@@ -96,9 +63,9 @@ int max_decompose_ctas(const PlanOps* ops) {
 bool layout_of(const PlanOps* ops, WsLayout* L) {
   const size_t n = (size_t)ops->n;
   L->status = 0;
-  L->tw = kAlign;
-  L->eps = L->tw + align_up(2 * n * sizeof(float2));
-  L->uslots = L->eps + align_up(((n + 31) / 32) * sizeof(uint32_t));
+  L->eps = kAlign;
+  L->tw = L->eps + align_up(((n + 31) / 32) * sizeof(uint32_t));
+  L->uslots = L->tw + align_up((size_t)ops->twn * sizeof(float2));
   size_t us = 0;
   if (ops->u_in_gmem) {
     const int ctas = max_decompose_ctas(ops);
@@ -111,13 +78,9 @@ bool layout_of(const PlanOps* ops, WsLayout* L) {
 
 kd_status setup(const PlanOps* ops, const WsLayout& L, void* ws, uint64_t seed, cudaStream_t s) {
   char* b = static_cast<char*>(ws);
-  const int n = ops->n;
-  const int threads = 256;
-  const int blocks = (2 * n + threads - 1) / threads;
-  setup_tables_kernel<<<blocks, threads, 0, s>>>(reinterpret_cast<float2*>(b + L.tw),
-                                                 reinterpret_cast<uint32_t*>(b + L.eps),
-                                                 reinterpret_cast<uint32_t*>(b + L.status), n, seed);
-  return cudaGetLastError() == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+  cudaError_t e = ops->setup(reinterpret_cast<float2*>(b + L.tw), reinterpret_cast<uint32_t*>(b + L.eps),
+                             reinterpret_cast<uint32_t*>(b + L.status), seed, s);
+  return e == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
 int grid_for(int64_t npairs, int q, int ctas_max) {
@@ -204,7 +167,7 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
   p.vhat = vhat;
   p.resid = resid;
   p.trace = trace;
-  p.tw = reinterpret_cast<const float2*>(b + L.tw);
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.status = reinterpret_cast<uint32_t*>(b + L.status);
   p.uslots = ops->u_in_gmem ? reinterpret_cast<float2*>(b + L.uslots) : nullptr;
@@ -232,7 +195,7 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
   p.x = x;
   p.y = y;
   p.m = m;
-  p.tw = reinterpret_cast<const float2*>(b + L.tw);
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.npairs = (m + 1) / 2;
   const int per = ops->ctas_per_sm(1);
@@ -268,7 +231,7 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
   p.m = m;
   p.ld = ld;
   p.out = w_hat;
-  p.tw = reinterpret_cast<const float2*>(b + L.tw);
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.npairs = (m + 1) / 2;
   const int per = ops->ctas_per_sm(2);

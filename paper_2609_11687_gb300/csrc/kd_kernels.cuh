@@ -28,67 +28,23 @@
 #pragma once
 
 #include <cstdint>
+#include <type_traits>
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include "kd_math.cuh"
+#include "kd_xform.cuh"
 
 namespace kd {
 
-enum { UREG = 0, UGMEM = 1 };
 enum { DT_F32 = 0, DT_F16 = 1, DT_BF16 = 2 };
 enum { LAY_ROWS = 0, LAY_COLS = 1 };
-
-// ---------------------------------------------------------------------------
-// Plan: radices R0..R{P-1} of the N-point FFT, team size T = N / R0, Q teams per
-// CTA, storage mode of u.
-// ---------------------------------------------------------------------------
-template <int N_, int T_, int Q_, int UMODE_, int MINB_, int... Rs>
-struct Plan {
-  static constexpr int N = N_;
-  static constexpr int MINB = MINB_;  // CTAs per SM the register budget must allow
-  static constexpr int T = T_;
-  static constexpr int Q = Q_;
-  static constexpr int UMODE = UMODE_;
-  static constexpr int NP = sizeof...(Rs);
-  static constexpr int Rv[NP] = {Rs...};
-  static constexpr int E = Rv[0];
-  static constexpr int THREADS = T * Q;
-  static constexpr int NW = (T + 31) / 32;           // warps per team
-  static constexpr int BUF = (N + N / 16 + 8 + 15) / 16 * 16;  // padded float2 slots per team (16-B aligned)
-  static constexpr int RED = 4 * (NW > 1 ? NW : 1);  // float2 reduction slots per team
-  static constexpr size_t SMEM = (size_t)Q * (BUF + RED) * sizeof(float2);
-
-  KD_HD static constexpr int R(int i) { return Rv[i]; }
-  KD_HD static constexpr int B(int i) {  // sub-transform length entering pass i
-    int b = N;
-    for (int j = 0; j < i; ++j) b /= Rv[j];
-    return b;
-  }
-  KD_HD static constexpr bool valid() {
-    int p = 1;
-    for (int i = 0; i < NP; ++i) p *= Rv[i];
-    return p == N && N == T * E && (N % 2 == 0) && NP >= 2 && (T <= 32 ? (32 % T == 0) : (T % 32 == 0 && Q == 1));
-  }
-  static_assert(valid(), "inconsistent plan");
-};
-
-__device__ __forceinline__ int pad(int i) { return i + (i >> 4); }
 
 // Natural index of Makhoul position p (N even).
 template <int N>
 __device__ __forceinline__ int nat_of(int p) {
   return (p < N / 2) ? 2 * p : 2 * N - 1 - 2 * p;
-}
-
-template <class PL>
-__device__ __forceinline__ void team_sync() {
-  if constexpr (PL::T <= 32) {
-    __syncwarp();
-  } else {
-    __syncthreads();
-  }
 }
 
 // Sum of v over the team; every thread receives the identical result.
@@ -114,138 +70,19 @@ __device__ __forceinline__ float2 team_sum(float2 v, float2* red, int lt, int& p
   }
 }
 
-// ---------------------------------------------------------------------------
-// Radix passes.  tw[j] = exp(-i pi j / N), j < 2N  (W_{2N}^j).
-// Pass i over sub-transforms of length B = B(i): group g -> block g / S, offset
-// np = g % S (S = B / R); elements at block*B + np + j*S.  Forward: radix-R DFT,
-// then twiddle W_B^{np*j} (none on the last pass).  Inverse: conjugate twiddle,
-// then inverse DFT, same slots.
-// ---------------------------------------------------------------------------
-template <class PL, int I, int DIR>
-__device__ __forceinline__ void pass_smem(float2* __restrict__ buf, const float2* __restrict__ tw, int lt) {
-  constexpr int R = PL::R(I);
-  constexpr int Bk = PL::B(I);
-  constexpr int S = Bk / R;
-  constexpr int G = PL::N / R;
-  constexpr bool LAST = (I == PL::NP - 1);
-  constexpr int TWS = 2 * PL::N / Bk;
-  for (int g = lt; g < G; g += PL::T) {
-    const int blk = g / S;
-    const int np = g - blk * S;
-    const int base = blk * Bk + np;
-    float2 v[R];
-#pragma unroll
-    for (int j = 0; j < R; ++j) v[j] = buf[pad(base + j * S)];
-    if constexpr (DIR < 0) {
-      Dft<R, -1>::run(v);
-      if constexpr (!LAST) {
-#pragma unroll
-        for (int j = 1; j < R; ++j) v[j] = cmul(v[j], __ldg(&tw[np * j * TWS]));
-      }
-    } else {
-      if constexpr (!LAST) {
-#pragma unroll
-        for (int j = 1; j < R; ++j) v[j] = cmulc(v[j], __ldg(&tw[np * j * TWS]));
-      }
-      Dft<R, +1>::run(v);
-    }
-#pragma unroll
-    for (int j = 0; j < R; ++j) buf[pad(base + j * S)] = v[j];
-  }
-}
-
-// Digit-reversed slot of frequency k: k = k0 + R0 k1 + R0 R1 k2 + ...  ->
-// slot = k0 (N/R0) + k1 (N/(R0 R1)) + ...
+// Shared memory of a CTA: [twiddle table (if staged)][team 0 buffer | red][team 1 ...].
+// Copies the table in and returns this team's buffer.
 template <class PL>
-__device__ __forceinline__ int slot_of(int k) {
-  int s = 0;
-  int rem = k;
-  static_for<0, PL::NP>([&](auto ii) {
-    constexpr int I = decltype(ii)::value;
-    constexpr int Ri = PL::R(I);
-    constexpr int stride = PL::B(I) / Ri;
-    const int ki = rem % Ri;
-    rem /= Ri;
-    s += ki * stride;
-  });
-  return s;
-}
-
-__device__ __forceinline__ float eps_of(const uint32_t* __restrict__ eb, int k) {
-  return ((__ldg(&eb[k >> 5]) >> (k & 31)) & 1u) ? -1.f : 1.f;
-}
-
-// The middle operator M (with the 1/N of the inverse DFT folded in).
-template <class PL>
-__device__ __forceinline__ void middle(float2* __restrict__ buf, const float2* __restrict__ tw,
-                                       const uint32_t* __restrict__ eb, int lt) {
-  constexpr int N = PL::N;
-  const float invN = 1.0f / (float)N;
-  for (int i = lt; i <= N / 2; i += PL::T) {
-    if (i == 0 || i == N / 2) {
-      const int s = pad(slot_of<PL>(i));
-      buf[s] = cscale(buf[s], eps_of(eb, i) * invN);
-    } else {
-      const int sa = pad(slot_of<PL>(i));
-      const int sb = pad(slot_of<PL>(N - i));
-      const float2 a = buf[sa];
-      const float2 b = buf[sb];
-      const float ek = eps_of(eb, i);
-      const float ekb = eps_of(eb, N - i);
-      float2 na, nb;
-      if (ek == ekb) {
-        const float f = ek * invN;
-        na = cscale(a, f);
-        nb = cscale(b, f);
-      } else {
-        // w = exp(+i pi k / N) = conj(tw[k]);  Z'_k = ek w Z_{N-k};  Z'_{N-k} = ek conj(w) Z_k
-        const float2 t = __ldg(&tw[i]);
-        const float f = ek * invN;
-        na = cscale(cmulc(b, t), f);
-        nb = cscale(cmul(a, t), f);
-      }
-      buf[sa] = na;
-      buf[sb] = nb;
-    }
+__device__ __forceinline__ float2* cta_setup(float2* smem, const float2* __restrict__ twg, const float2*& tw,
+                                             int team) {
+  if constexpr (PL::TW_SMEM) {
+    for (int i = threadIdx.x; i < PL::TWN; i += blockDim.x) smem[i] = __ldg(&twg[i]);
+    __syncthreads();
+    tw = smem;
+  } else {
+    tw = twg;
   }
-}
-
-// y = P' v for the team's vector pair held in registers (E values per thread).
-template <class PL>
-__device__ __forceinline__ void apply_P(float2 (&v)[PL::E], float2* __restrict__ buf,
-                                        const float2* __restrict__ tw, const uint32_t* __restrict__ eb,
-                                        int lt) {
-  constexpr int E = PL::E;
-  constexpr int T = PL::T;
-  if constexpr (PL::T <= 32) team_sync<PL>();  // previous readers of buf are done
-  // forward pass 0 from registers: group np = lt, stride T, twiddle W_N^{lt*j} = tw[2*lt*j]
-  Dft<E, -1>::run(v);
-#pragma unroll
-  for (int j = 0; j < E; ++j) {
-    float2 x = v[j];
-    if (j > 0) x = cmul(x, __ldg(&tw[2 * lt * j]));
-    buf[pad(lt + j * T)] = x;
-  }
-  team_sync<PL>();
-  static_for<1, PL::NP>([&](auto ii) {
-    constexpr int I = decltype(ii)::value;
-    pass_smem<PL, I, -1>(buf, tw, lt);
-    team_sync<PL>();
-  });
-  middle<PL>(buf, tw, eb, lt);
-  team_sync<PL>();
-  static_for<1, PL::NP>([&](auto ii) {
-    constexpr int I = PL::NP - decltype(ii)::value;
-    pass_smem<PL, I, +1>(buf, tw, lt);
-    team_sync<PL>();
-  });
-#pragma unroll
-  for (int j = 0; j < E; ++j) {
-    float2 x = buf[pad(lt + j * T)];
-    if (j > 0) x = cmulc(x, __ldg(&tw[2 * lt * j]));
-    v[j] = x;
-  }
-  Dft<E, +1>::run(v);
+  return smem + PL::SMEM_TW / sizeof(float2) + team * PL::TEAM;
 }
 
 // ---------------------------------------------------------------------------
@@ -293,7 +130,7 @@ struct DecParams {
   float* vhat;
   float* resid;
   int8_t* trace;
-  const float2* tw;
+  const float2* twt;      // access-ordered twiddle table (global)
   const uint32_t* eps;
   uint32_t* status;
   float2* uslots;
@@ -308,7 +145,7 @@ __device__ __forceinline__ float signed_step(float r, float c) {
 // ---------------------------------------------------------------------------
 // kd_decompose kernel
 // ---------------------------------------------------------------------------
-template <class PL>
+template <class PL, bool TRACE>
 __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecParams p) {
   constexpr int N = PL::N;
   constexpr int T = PL::T;
@@ -316,14 +153,19 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
   extern __shared__ __align__(16) float2 smem[];
   const int team = threadIdx.x / T;
   const int lt = threadIdx.x - team * T;
-  float2* buf = smem + team * (PL::BUF + PL::RED);
+  const float2* tw;
+  float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
   float2* red = buf + PL::BUF;
+  Xform<PL> xf;
+  xf.init(buf, tw, p.eps, lt);
   int parity = 0;
   const int nsteps = 4 * p.iters;
 
   float2 uu_reg[PL::UMODE == UREG ? E : 1];
+  // u outside registers: per-team workspace slot (global) or shared memory after red
   float2* uslot = nullptr;
   if constexpr (PL::UMODE == UGMEM) uslot = p.uslots + ((int64_t)blockIdx.x * PL::Q + team) * N;
+  if constexpr (PL::UMODE == USMEM) uslot = red + PL::RED;
 
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
@@ -380,10 +222,10 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
 #pragma unroll
     for (int q = 0; q < 4; ++q) coef[q] = make_float2(0.f, 0.f);
 
-    const bool tracing = (p.trace != nullptr) && active;
+    const bool tracing = TRACE && active;
     int8_t* trA = nullptr;
     int8_t* trB = nullptr;
-    if (tracing) {
+    if (TRACE && tracing) {
       trA = p.trace + colA * (int64_t)nsteps * N;
       trB = p.trace + colB * (int64_t)nsteps * N;
     }
@@ -405,7 +247,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
       const float lB = __fdiv_rn(s.y, (float)N);
 #pragma unroll
       for (int j = 0; j < E; ++j) {
-        if (tracing) {
+        if (TRACE && tracing) {
           const int nat = nat_of<N>(lt + j * T);
           const int64_t off = (int64_t)step * N + nat;
           trA[off] = (int8_t)((r[j].x > 0.f) - (r[j].x < 0.f));
@@ -429,36 +271,46 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
 
     int step = 0;
     for (int t = 0; t < p.iters; ++t) {
-      // two greedy steps from Q_N (update u)
-      float2 ugm[PL::UMODE == UGMEM ? E : 1];
-      if constexpr (PL::UMODE == UGMEM) {
-#pragma unroll
-        for (int j = 0; j < E; ++j) ugm[j] = uslot[lt + j * T];
-      }
-      auto add_u_any = [&](int j, float dA, float dB) {
+      // two greedy steps from Q_N (update u).  With u outside registers, step 1's
+      // signs are kept as bits and u is updated once after step 2 as
+      // (u + d1) + d2 -- the same roundings as two separate updates.
+      using Bits = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
+      Bits nzA = 0, ngA = 0, nzB = 0, ngB = 0;
+      float2 l1 = make_float2(0.f, 0.f);
+      auto rec1 = [&](int j, float dA, float dB) {
         if constexpr (PL::UMODE == UREG) {
           add_u(j, dA, dB);
         } else {
-          ugm[j].x = __fadd_rn(ugm[j].x, dA);
-          ugm[j].y = __fadd_rn(ugm[j].y, dB);
+          nzA |= (Bits)(dA != 0.f) << j;
+          ngA |= (Bits)(dA < 0.f) << j;
+          nzB |= (Bits)(dB != 0.f) << j;
+          ngB |= (Bits)(dB < 0.f) << j;
         }
       };
-      float2 l1 = greedy(step, t == 0, sum0, add_u_any);
+      auto upd2 = [&](int j, float dA, float dB) {
+        if constexpr (PL::UMODE == UREG) {
+          add_u(j, dA, dB);
+        } else {
+          const float d1A = ((nzA >> j) & 1u) ? (((ngA >> j) & 1u) ? -l1.x : l1.x) : 0.f;
+          const float d1B = ((nzB >> j) & 1u) ? (((ngB >> j) & 1u) ? -l1.y : l1.y) : 0.f;
+          float2 uj = uslot[lt + j * T];
+          uj.x = __fadd_rn(__fadd_rn(uj.x, d1A), dA);
+          uj.y = __fadd_rn(__fadd_rn(uj.y, d1B), dB);
+          uslot[lt + j * T] = uj;
+        }
+      };
+      l1 = greedy(step, t == 0, sum0, rec1);
       ++step;
-      float2 l2 = greedy(step, false, sum0, add_u_any);
+      float2 l2 = greedy(step, false, sum0, upd2);
       ++step;
-      if constexpr (PL::UMODE == UGMEM) {
-#pragma unroll
-        for (int j = 0; j < E; ++j) uslot[lt + j * T] = ugm[j];
-      }
       // two greedy steps from P Q_N on y = P rho (update vhat implicitly)
-      apply_P<PL>(r, buf, p.tw, p.eps, lt);
+      xf.apply(r);
       mask_dead(r);
       float2 l3 = greedy(step, false, sum0, add_none);
       ++step;
       float2 l4 = greedy(step, false, sum0, add_none);
       ++step;
-      apply_P<PL>(r, buf, p.tw, p.eps, lt);
+      xf.apply(r);
       mask_dead(r);
       if (t == 0) {
         coef[0] = l1;
@@ -468,46 +320,54 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
       }
     }
 
-    // ---- vhat = P (x - u - r) ----
+    // ---- residual out, then vhat = P (x - u - r) ----
+    const float isA = pow2f(-sA), isB = pow2f(-sB);
+    if (active && p.resid) {
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        const int nat = nat_of<N>(lt + j * T);
+        p.resid[colA * N + nat] = __fmul_rn(r[j].x, isA);
+        if (hasB) p.resid[colB * N + nat] = __fmul_rn(r[j].y, isB);
+      }
+    }
+    auto u_at = [&](int j) -> float2 {
+      if constexpr (PL::UMODE == UREG) {
+        return uu_reg[j];
+      } else {
+        return uslot[lt + j * T];
+      }
+    };
     float2 vh[E];
-    float2 uf[E];
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
       const float a = __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld)), scA);
       const float b = hasB ? __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)), scB) : 0.f;
-      if constexpr (PL::UMODE == UREG) {
-        uf[j] = uu_reg[j];
-      } else {
-        uf[j] = uslot[lt + j * T];
-      }
-      vh[j] = make_float2(__fsub_rn(__fsub_rn(a, uf[j].x), r[j].x), __fsub_rn(__fsub_rn(b, uf[j].y), r[j].y));
+      const float2 uj = u_at(j);
+      vh[j] = make_float2(__fsub_rn(__fsub_rn(a, uj.x), r[j].x), __fsub_rn(__fsub_rn(b, uj.y), r[j].y));
     }
     if (p.iters > 0) {
-      apply_P<PL>(vh, buf, p.tw, p.eps, lt);
+      team_sync<PL>();  // the last transform's readers of buf are done
+      xf.apply(vh);
       mask_dead(vh);
     } else {
 #pragma unroll
       for (int j = 0; j < E; ++j) vh[j] = make_float2(0.f, 0.f);
     }
 
-    // ---- optional dense outputs (natural order, scaled back) ----
-    const float isA = pow2f(-sA), isB = pow2f(-sB);
-    if (active) {
+    // ---- optional dense factors (natural order, scaled back) ----
+    if (active && (p.u || p.vhat)) {
 #pragma unroll
       for (int j = 0; j < E; ++j) {
         const int nat = nat_of<N>(lt + j * T);
+        const float2 uj = u_at(j);
         if (p.u) {
-          p.u[colA * N + nat] = __fmul_rn(uf[j].x, isA);
-          if (hasB) p.u[colB * N + nat] = __fmul_rn(uf[j].y, isB);
+          p.u[colA * N + nat] = __fmul_rn(uj.x, isA);
+          if (hasB) p.u[colB * N + nat] = __fmul_rn(uj.y, isB);
         }
         if (p.vhat) {
           p.vhat[colA * N + nat] = __fmul_rn(vh[j].x, isA);
           if (hasB) p.vhat[colB * N + nat] = __fmul_rn(vh[j].y, isB);
-        }
-        if (p.resid) {
-          p.resid[colA * N + nat] = __fmul_rn(r[j].x, isA);
-          if (hasB) p.resid[colB * N + nat] = __fmul_rn(r[j].y, isB);
         }
       }
     }
@@ -523,8 +383,9 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
       auto code = [](float x, float mm) -> uint8_t {
         return (uint8_t)((x > -mm) + (x > 0.f) + (x > mm));
       };
-      cb[0 * N + nat] = code(uf[j].x, muA);
-      cb[1 * N + nat] = code(uf[j].y, muB);
+      const float2 uj = u_at(j);
+      cb[0 * N + nat] = code(uj.x, muA);
+      cb[1 * N + nat] = code(uj.y, muB);
       cb[2 * N + nat] = code(vh[j].x, mvA);
       cb[3 * N + nat] = code(vh[j].y, mvB);
     }
@@ -581,7 +442,7 @@ struct ApplyParams {
   const float* x;
   float* y;
   int64_t m;
-  const float2* tw;
+  const float2* twt;
   const uint32_t* eps;
   int64_t npairs;
 };
@@ -594,7 +455,10 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyPar
   extern __shared__ __align__(16) float2 smem[];
   const int team = threadIdx.x / T;
   const int lt = threadIdx.x - team * T;
-  float2* buf = smem + team * (PL::BUF + PL::RED);
+  const float2* tw;
+  float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
+  Xform<PL> xf;
+  xf.init(buf, tw, p.eps, lt);
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
     const bool active = pair < p.npairs;
@@ -608,7 +472,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyPar
       v[j] = make_float2(__ldg(&p.x[colA * N + nat]), hasB ? __ldg(&p.x[(colA + 1) * N + nat]) : 0.f);
     }
     team_sync<PL>();  // x and y may alias: all loads of this pair precede any store
-    apply_P<PL>(v, buf, p.tw, p.eps, lt);
+    xf.apply(v);
     if (active) {
 #pragma unroll
       for (int j = 0; j < E; ++j) {
@@ -632,7 +496,7 @@ struct RecParams {
   const float* centres_v;
   int64_t m, ld;
   void* out;
-  const float2* tw;
+  const float2* twt;
   const uint32_t* eps;
   int64_t npairs;
 };
@@ -646,7 +510,10 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
   extern __shared__ __align__(16) float2 smem[];
   const int team = threadIdx.x / T;
   const int lt = threadIdx.x - team * T;
-  float2* buf = smem + team * (PL::BUF + PL::RED);
+  const float2* tw;
+  float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
+  Xform<PL> xf;
+  xf.init(buf, tw, p.eps, lt);
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
     const bool active = pair < p.npairs;
@@ -673,7 +540,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
       uq[j] = make_float2(ua, ub);
       vq[j] = make_float2(va, vb);
     }
-    apply_P<PL>(vq, buf, p.tw, p.eps, lt);
+    xf.apply(vq);
     if (active) {
 #pragma unroll
       for (int j = 0; j < E; ++j) {

@@ -25,7 +25,7 @@ inline int occupancy(K kernel, int threads, size_t smem) {
 template <class PL>
 struct Ops {
   static cudaError_t decompose(const DecParams& p, int grid, cudaStream_t s) {
-    auto k = decompose_kernel<PL>;
+    auto k = p.trace ? decompose_kernel<PL, true> : decompose_kernel<PL, false>;
     cudaError_t e = prepare(k, PL::SMEM);
     if (e != cudaSuccess) return e;
     k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
@@ -45,14 +45,21 @@ struct Ops {
     k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
     return cudaGetLastError();
   }
+  static cudaError_t setup(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, cudaStream_t s) {
+    constexpr int threads = 256;
+    constexpr int work = PL::TWN > (PL::N + 31) / 32 ? PL::TWN : (PL::N + 31) / 32;
+    constexpr int blocks = (work + threads - 1) / threads;
+    setup_kernel<PL><<<blocks, threads, 0, s>>>(twt, eps, status, seed);
+    return cudaGetLastError();
+  }
   static int ctas_per_sm(int which) {
-    if (which == 0) return occupancy(decompose_kernel<PL>, PL::THREADS, PL::SMEM);
+    if (which == 0) return occupancy(decompose_kernel<PL, false>, PL::THREADS, PL::SMEM);
     if (which == 1) return occupancy(apply_p_kernel<PL>, PL::THREADS, PL::SMEM);
     return occupancy(reconstruct_kernel<PL>, PL::THREADS, PL::SMEM);
   }
   static const PlanOps* ops() {
-    static const PlanOps o{PL::N, PL::THREADS, PL::Q, PL::SMEM, PL::UMODE == UGMEM,
-                           &Ops::ctas_per_sm, &Ops::decompose, &Ops::apply, &Ops::reconstruct};
+    static const PlanOps o{PL::N, PL::THREADS, PL::Q, PL::SMEM, PL::UMODE == UGMEM, PL::TWN,
+                           &Ops::ctas_per_sm, &Ops::decompose, &Ops::apply, &Ops::reconstruct, &Ops::setup};
     return &o;
   }
 };

@@ -228,6 +228,56 @@ struct DftPrime {
   }
 };
 
+// Odd prime R, streaming form: inputs come from load(n) (each read once), outputs
+// leave through store(k, X) as soon as they are formed, so only the symmetric
+// sums a_n, b_n stay live (used where R is too large to hold inputs and outputs
+// in registers at once).
+template <int R, int DIR, class Load, class Store>
+__device__ __forceinline__ void dft_prime_stream(Load&& load, Store&& store) {
+  constexpr int H = (R - 1) / 2;
+  float2 a[H + 1], b[H + 1];
+  const float2 x0 = load(0);
+  float2 sum = x0;
+#pragma unroll
+  for (int n = 1; n <= H; ++n) {
+    const float2 p = load(n), q = load(R - n);
+    a[n] = cadd(p, q);
+    b[n] = csub(p, q);
+    sum = cadd(sum, a[n]);
+  }
+  store(0, sum);
+  static_for<1, H + 1>([&](auto kk) {
+    constexpr int K = decltype(kk)::value;
+    float2 ak = x0;
+    float2 bk = make_float2(0.f, 0.f);
+    static_for<1, H + 1>([&](auto nn) {
+      constexpr int NN = decltype(nn)::value;
+      constexpr float c = (float)cos2pi((long long)NN * K, R);
+      constexpr float sn = (float)sin2pi((long long)NN * K, R);
+      ak.x = __fmaf_rn(a[NN].x, c, ak.x);
+      ak.y = __fmaf_rn(a[NN].y, c, ak.y);
+      bk.x = __fmaf_rn(b[NN].x, sn, bk.x);
+      bk.y = __fmaf_rn(b[NN].y, sn, bk.y);
+    });
+    const float2 ib = mul_pi(bk);
+    if constexpr (DIR < 0) {
+      store(K, csub(ak, ib));
+      store(R - K, cadd(ak, ib));
+    } else {
+      store(K, cadd(ak, ib));
+      store(R - K, csub(ak, ib));
+    }
+  });
+}
+
+template <int R>
+KD_HD constexpr bool kd_is_big_prime() {
+  if (R < 11 || R % 2 == 0) return false;
+  for (int d = 3; d * d <= R; d += 2)
+    if (R % d == 0) return false;
+  return true;
+}
+
 // Composite R = A * B (A = smallest factor, 4 preferred): decimation in frequency.
 //   n = B*n1 + n2 ; k = k1 + A*k2
 //   step 1: for each n2, size-A DFT over n1 -> k1 ; multiply by W_R^{n2*k1}

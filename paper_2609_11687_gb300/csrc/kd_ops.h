@@ -16,11 +16,14 @@ struct PlanOps {
   int q;            // vector pairs per CTA per iteration
   size_t smem;      // dynamic shared memory per CTA
   bool u_in_gmem;   // u lives in per-team workspace slots
+  int twn;          // entries of the access-ordered twiddle table
   // CTAs that fit on one SM (occupancy), 0 on error
   int (*ctas_per_sm)(int which);  // which: 0 decompose, 1 apply, 2 reconstruct
   cudaError_t (*decompose)(const DecParams&, int grid, cudaStream_t);
   cudaError_t (*apply)(const ApplyParams&, int grid, cudaStream_t);
   cudaError_t (*reconstruct)(const RecParams&, int grid, cudaStream_t);
+  // tables for one call: twiddles (float2[twn]), sign bits, cleared status word
+  cudaError_t (*setup)(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, cudaStream_t);
 };
 
 const PlanOps* plan_ops(int64_t n);

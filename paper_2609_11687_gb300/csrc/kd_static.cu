@@ -9,7 +9,7 @@
 // of a caller workspace, so it allocates nothing.
 //
 // Limits and sharing:
-//  - the array holds the tables of one vector length up to KD_STATIC_MAX_N (8192);
+//  - the array holds the tables of one vector length up to 8192;
 //    longer vectors are rejected with KD_ERR_WORKSPACE before anything is enqueued;
 //  - every GPU that loads the library holds the array until the process exits;
 //  - all calls share it and it keeps the last call's contents; each call rewrites
@@ -29,7 +29,7 @@ namespace kd {
 namespace {
 
 constexpr int64_t kStaticMaxN = 8192;
-constexpr size_t kStaticBytes = 160 * 1024;  // >= 256 + 16*8192 + 1024 (status, twiddles, sign bits)
+constexpr size_t kStaticBytes = 160 * 1024;  // >= kd_workspace_size(n) for every n <= 8192 (checked per call)
 constexpr int kMaxDevices = 64;
 
 // Host code must not pass `kd_static_scratch` itself to a kernel: on the host that

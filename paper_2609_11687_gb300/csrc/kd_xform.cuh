@@ -1,0 +1,434 @@
+// The sign-randomised DCT operator P on a pair of vectors held by one team
+// (Sec. 3.1: P z = IDCT(eps * DCT(z)); Alg. 1 applies it twice per block).
+//
+// With both vectors in Makhoul's even/odd order and packed as one complex
+// vector z (vector 2j in the real part, 2j+1 in the imaginary part),
+//     P' z = IDFT( M( DFT(z) ) ),
+//     M: Z'_k = e+_k Z_k + e-_k exp(i pi k/N) Z_{N-k},  e+-_k = (eps_k +- eps_{N-k}) / 2,
+// (the DCT's per-coefficient scale cancels between DCT and IDCT).  Exactly one of
+// e+_k, e-_k is non-zero: either Z'_k = eps_k Z_k, or Z'_k = eps_k exp(i pi k/N) Z_{N-k}.
+//
+// DFT: in-place mixed-radix decimation in frequency over shared memory (natural
+// order in, digit-reversed out); IDFT: the mirror passes (digit-reversed in,
+// natural out).  Pass 0 works on the thread's own registers (the vector stays
+// register-resident between transforms).  Inter-pass twiddles come from a table
+// laid out in the order the threads read it (conflict-free in shared memory).
+//
+// M runs in one of two forms:
+//  * paired (last radix == first radix, one last-pass group per thread): the
+//    thread owning frequency group K and the one owning N/R0 - K sit at lanes
+//    l and l ^ H of one warp; each gets its partner's values by shuffle and
+//    applies M in registers between the last forward and first inverse pass;
+//  * slot order (all other plans): each thread reads its own slots and their
+//    partners' from shared memory (conflict-free: partners of consecutive slots
+//    are consecutive slots in reverse), then writes its own.
+// All per-frequency quantities (partner slot, eps bits, exp(i pi k/N)) reduce to
+// a few per-thread constants computed once per CTA.
+#pragma once
+
+#include "kd_math.cuh"
+
+namespace kd {
+
+enum { UREG = 0, UGMEM = 1, USMEM = 2 };
+
+template <int N_, int T_, int Q_, int UMODE_, int MINB_, int... Rs>
+struct Plan {
+  static constexpr int N = N_;
+  static constexpr int T = T_;
+  static constexpr int Q = Q_;
+  static constexpr int UMODE = UMODE_;
+  static constexpr int MINB = MINB_;  // CTAs per SM the register budget must allow
+  static constexpr int NP = sizeof...(Rs);
+  static constexpr int Rv[NP] = {Rs...};
+  static constexpr int E = Rv[0];
+  static constexpr int RL = Rv[NP - 1];
+  static constexpr int THREADS = T * Q;
+  static constexpr int NW = (T + 31) / 32;  // warps per team
+  static constexpr int BUF = (N + N / 16 + 8 + 15) / 16 * 16;  // padded float2 slots per team
+  static constexpr int RED = 4 * (NW > 1 ? NW : 1);           // float2 reduction slots per team
+  static constexpr int USL = (UMODE_ == 2) ? N : 0;            // float2 slots of u per team (shared)
+  // M in registers: one last-pass group per thread, partner at lane ^ HALF
+#ifdef KD_NO_PAIRED
+  static constexpr bool PAIRED = false;
+#else
+  static constexpr bool PAIRED = (RL == E) && (N / RL == T);
+#endif
+  static constexpr int HALF = (T < 32 ? T : 32) / 2;
+
+  KD_HD static constexpr int R(int i) { return Rv[i]; }
+  KD_HD static constexpr int B(int i) {  // sub-transform length entering pass i
+    int b = N;
+    for (int j = 0; j < i; ++j) b /= Rv[j];
+    return b;
+  }
+  KD_HD static constexpr int S(int i) { return B(i) / Rv[i]; }  // stride of pass i's digit
+  // access-ordered twiddle table: pass 0 [j][t] (N entries), pass i>=1 [j][np] (B(i) entries)
+  KD_HD static constexpr int tw_off(int i) {
+    int o = 0;
+    for (int j = 0; j < i; ++j) o += B(j);
+    return o;
+  }
+  static constexpr int TWN = tw_off(NP - 1);
+  // stage the table in shared memory when MINB CTAs per SM still fit
+  static constexpr int TEAM = BUF + RED + USL;  // float2 slots of shared memory per team
+  static constexpr bool TW_SMEM = (size_t)TWN * 8 + (size_t)Q * TEAM * 8 <= (size_t)(227 * 1024) / MINB - 1024;
+  static constexpr size_t SMEM_TW = TW_SMEM ? (size_t)TWN * sizeof(float2) : 0;
+  static constexpr size_t SMEM = SMEM_TW + (size_t)Q * TEAM * sizeof(float2);
+
+  KD_HD static constexpr bool valid() {
+    int p = 1;
+    for (int i = 0; i < NP; ++i) p *= Rv[i];
+    return p == N && N == T * E && (N % 16 == 0) && NP >= 2 &&
+           (T <= 32 ? (32 % T == 0) : (T % 32 == 0 && Q == 1));
+  }
+  static_assert(valid(), "inconsistent plan");
+};
+
+__device__ __forceinline__ int pad(int i) { return i + (i >> 4); }
+
+// Twiddle read that the compiler may not hoist out of the block loop: every
+// thread's twiddles are loop-invariant, and keeping them all in registers would
+// spill.  SMEM selects a shared-memory (else read-only global) load.
+template <bool SMEM>
+__device__ __forceinline__ float2 ld_tw(const float2* p) {
+  float2 v;
+  if constexpr (SMEM) {
+    const unsigned a = (unsigned)__cvta_generic_to_shared(p);
+    asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
+  } else {
+    asm volatile("ld.global.nc.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(p));
+  }
+  return v;
+}
+
+template <class PL>
+__device__ __forceinline__ void team_sync() {
+  if constexpr (PL::T <= 32) {
+    __syncwarp();
+  } else {
+    __syncthreads();
+  }
+}
+
+__device__ __forceinline__ bool eps_neg(const uint32_t* __restrict__ eb, int k) {
+  return (__ldg(&eb[k >> 5]) >> (k & 31)) & 1u;
+}
+
+// exp(i pi a / b) in double, rounded
+__device__ __forceinline__ float2 expi_pi(long long a, long long b) {
+  double s, c;
+  sincospi((double)a / (double)b, &s, &c);
+  return make_float2((float)c, (float)s);
+}
+
+// Digit-reversed slot of X over passes 1..NP-1: X = sum x_i prod_{1<=j<i} R_j  ->  sum x_i S_i
+template <class PL>
+__device__ __forceinline__ int slot_rest(int X) {
+  int s = 0;
+  static_for<1, PL::NP>([&](auto ii) {
+    constexpr int I = decltype(ii)::value;
+    const int xi = X % PL::R(I);
+    X /= PL::R(I);
+    s += xi * PL::S(I);
+  });
+  return s;
+}
+
+// Slot of the first element of the last-pass group that holds frequencies
+// K + (N/RL) j: the digits of K over passes 0..NP-2 placed at their strides.
+template <class PL>
+__device__ __forceinline__ int slot_low(int K) {
+  int s = 0;
+  static_for<0, PL::NP - 1>([&](auto ii) {
+    constexpr int I = decltype(ii)::value;
+    const int ki = K % PL::R(I);
+    K /= PL::R(I);
+    s += ki * PL::S(I);
+  });
+  return s;
+}
+
+// Inverse of slot_rest for a slot below T (digits of passes 1..NP-1).
+template <class PL>
+__device__ __forceinline__ int rest_of_slot(int s) {
+  int X = 0, mul = 1;
+  static_for<1, PL::NP>([&](auto ii) {
+    constexpr int I = decltype(ii)::value;
+    const int xi = (s / PL::S(I)) % PL::R(I);
+    X += xi * mul;
+    mul *= PL::R(I);
+  });
+  return X;
+}
+
+// ---------------------------------------------------------------------------
+template <class PL>
+struct Xform {
+  static constexpr int N = PL::N, T = PL::T, E = PL::E, NP = PL::NP;
+  float2* buf;                 // team's padded exchange buffer (shared)
+  const float2* tw;            // access-ordered twiddles (shared or global)
+  int lt;
+  float2 cw;                   // M twiddle base
+  using Mask = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
+  Mask ek, em;                 // eps_k < 0 / eps_{-k} < 0 for each owned frequency (bit index)
+  int p0, p1;                  // slot-order M: partner slot constants
+  int kgrp;                    // paired M: own frequency group (k = kgrp + (N/RL) j)
+  int lbase;                   // paired M: slot of that group's first element
+  int self;                    // paired M: 0 regular, 1 group 0, 2 group N/(2 R0)
+
+  __device__ __forceinline__ void init(float2* b, const float2* t, const uint32_t* __restrict__ eb, int lane_t) {
+    buf = b;
+    tw = t;
+    lt = lane_t;
+    ek = em = 0;
+    if constexpr (PL::PAIRED) {
+      constexpr int H = PL::HALF;
+      constexpr int L = T;
+      const int w = lt / (2 * H), l = lt % (2 * H), h = l / H, i = l % H;
+      const int bb = H * w + i;
+      kgrp = h ? (bb ? L - bb : L / 2) : bb;
+      self = (bb == 0) ? (h == 0 ? 1 : 2) : 0;
+      lbase = slot_low<PL>(kgrp);
+      cw = expi_pi(kgrp, N);
+#pragma unroll
+      for (int kp = 0; kp < E; ++kp) {
+        const int k = kgrp + L * kp;
+        ek |= (Mask)eps_neg(eb, k) << kp;
+        em |= (Mask)eps_neg(eb, (N - k) % N) << kp;
+      }
+      p0 = p1 = 0;
+    } else {
+      const int Kp = rest_of_slot<PL>(lt);
+      p0 = slot_rest<PL>((T - Kp) % T);
+      p1 = slot_rest<PL>(T - 1 - Kp);
+      cw = expi_pi((long long)E * Kp, N);
+#pragma unroll
+      for (int r = 0; r < E; ++r) {
+        const int k = r + E * Kp;
+        ek |= (Mask)eps_neg(eb, k) << r;
+        em |= (Mask)eps_neg(eb, (N - k) % N) << r;
+      }
+      kgrp = self = lbase = 0;
+    }
+  }
+
+  // M on one frequency: own value a, partner value b; returns Z'_k (1/N folded in).
+  template <long long RNUM, long long RDEN>
+  __device__ __forceinline__ float2 mfreq(float2 a, float2 b, int bit) const {
+    constexpr float invN = 1.0f / (float)N;
+    const bool neg = (ek >> bit) & 1u;
+    const bool negm = (em >> bit) & 1u;
+    const float f = neg ? -invN : invN;
+    // exp(i pi k / N) = cw * exp(i pi RNUM / RDEN)
+    const float2 wk = mul_root<+1, RNUM, 2 * RDEN>(cw);
+    const float2 t = cmul(b, wk);
+    const float2 sel = (neg == negm) ? a : t;
+    return cscale(sel, f);
+  }
+
+  // forward pass 0 from registers
+  __device__ __forceinline__ void fwd0(float2 (&v)[E]) {
+    if constexpr (kd_is_big_prime<E>()) {
+      dft_prime_stream<E, -1>([&](int j) { return v[j]; },
+                              [&](int k, float2 x) {
+                                if (k > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + k * T + lt));
+                                buf[pad(lt + k * T)] = x;
+                              });
+    } else {
+      Dft<E, -1>::run(v);
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        float2 x = v[j];
+        if (j > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + j * T + lt));
+        buf[pad(lt + j * T)] = x;
+      }
+    }
+  }
+
+  // inverse pass 0 into registers
+  __device__ __forceinline__ void inv0(float2 (&v)[E]) {
+    if constexpr (kd_is_big_prime<E>()) {
+      // outputs go back to the thread's own slots (already read), then to registers
+      dft_prime_stream<E, +1>(
+          [&](int j) {
+            float2 x = buf[pad(lt + j * T)];
+            if (j > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + j * T + lt));
+            return x;
+          },
+          [&](int k, float2 x) { buf[pad(lt + k * T)] = x; });
+#pragma unroll
+      for (int j = 0; j < E; ++j) v[j] = buf[pad(lt + j * T)];
+    } else {
+#pragma unroll
+      for (int j = 0; j < E; ++j) {
+        float2 x = buf[pad(lt + j * T)];
+        if (j > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + j * T + lt));
+        v[j] = x;
+      }
+      Dft<E, +1>::run(v);
+    }
+  }
+
+  // shared-memory pass I (1 <= I <= NP-1), forward (DIR < 0) or inverse
+  template <int I, int DIR>
+  __device__ __forceinline__ void pass() {
+    constexpr int R = PL::R(I);
+    constexpr int Bk = PL::B(I);
+    constexpr int S = Bk / R;
+    constexpr int G = N / R;
+    constexpr bool LAST = (I == NP - 1);
+    constexpr int OFF = PL::tw_off(I);
+    for (int g = lt; g < G; g += T) {
+      const int blk = g / S;
+      const int np = g - blk * S;
+      const int base = blk * Bk + np;
+      float2 v[R];
+#pragma unroll
+      for (int j = 0; j < R; ++j) v[j] = buf[pad(base + j * S)];
+      if constexpr (DIR < 0) {
+        Dft<R, -1>::run(v);
+        if constexpr (!LAST) {
+#pragma unroll
+          for (int j = 1; j < R; ++j) v[j] = cmul(v[j], ld_tw<PL::TW_SMEM>(tw + OFF + j * S + np));
+        }
+      } else {
+        if constexpr (!LAST) {
+#pragma unroll
+          for (int j = 1; j < R; ++j) v[j] = cmulc(v[j], ld_tw<PL::TW_SMEM>(tw + OFF + j * S + np));
+        }
+        Dft<R, +1>::run(v);
+      }
+#pragma unroll
+      for (int j = 0; j < R; ++j) buf[pad(base + j * S)] = v[j];
+    }
+  }
+
+  // paired last pass: forward DFT of own group, M with the partner lane, inverse DFT
+  __device__ __forceinline__ void last_paired() {
+    constexpr int R = PL::RL;
+    constexpr int H = PL::HALF;
+    const int base = lbase;
+    float2 v[R];
+#pragma unroll
+    for (int j = 0; j < R; ++j) v[j] = buf[pad(base + j)];
+    Dft<R, -1>::run(v);
+    float2 o[R];
+    static_for<0, R>([&](auto kk) {
+      constexpr int KP = decltype(kk)::value;
+      const float2 src = v[R - 1 - KP];
+      float2 q;
+      q.x = __shfl_xor_sync(0xffffffffu, src.x, H);
+      q.y = __shfl_xor_sync(0xffffffffu, src.y, H);
+      if (self == 1) q = v[(R - KP) % R];
+      else if (self == 2) q = v[R - 1 - KP];
+      // k = K + (N/R) KP: exp(i pi k/N) = exp(i pi K/N) exp(i pi KP/R)
+      o[KP] = mfreq<KP, R>(v[KP], q, KP);
+    });
+    Dft<R, +1>::run(o);
+#pragma unroll
+    for (int j = 0; j < R; ++j) buf[pad(base + j)] = o[j];
+  }
+
+  // slot-order M (own slots lt + T r, partners from constants); v is scratch
+  __device__ __forceinline__ void middle_slots(float2 (&v)[E]) {
+    static_for<0, E>([&](auto rr) {
+      constexpr int RR = decltype(rr)::value;
+      const int s = lt + T * RR;
+      const int ps = (RR == 0) ? p0 : (E - RR) * T + p1;
+      // k = RR + E K': exp(i pi k/N) = exp(i pi E K'/N) exp(i pi RR/N)
+      v[RR] = mfreq<RR, N>(buf[pad(s)], buf[pad(ps)], RR);
+    });
+    team_sync<PL>();
+#pragma unroll
+    for (int r = 0; r < E; ++r) buf[pad(lt + T * r)] = v[r];
+  }
+
+  // y = P' v
+  __device__ __forceinline__ void apply(float2 (&v)[E]) {
+    if constexpr (T <= 32) team_sync<PL>();  // earlier readers of buf are done
+    fwd0(v);
+    team_sync<PL>();
+    if constexpr (PL::PAIRED) {
+      static_for<1, NP - 1>([&](auto ii) {
+        pass<decltype(ii)::value, -1>();
+        team_sync<PL>();
+      });
+      last_paired();
+      team_sync<PL>();
+      static_for<1, NP - 1>([&](auto ii) {
+        pass<NP - 1 - decltype(ii)::value, +1>();
+        team_sync<PL>();
+      });
+    } else {
+      static_for<1, NP>([&](auto ii) {
+        pass<decltype(ii)::value, -1>();
+        team_sync<PL>();
+      });
+      middle_slots(v);
+      team_sync<PL>();
+      static_for<1, NP>([&](auto ii) {
+        pass<NP - decltype(ii)::value, +1>();
+        team_sync<PL>();
+      });
+    }
+    inv0(v);
+  }
+};
+
+// ---------------------------------------------------------------------------
+// Table set-up for one plan: access-ordered twiddles (double-precision sincospi,
+// rounded), the sign bits (SplitMix64 of seed + (j+1)*gamma, bit 63 set ->
+// eps_j = -1) and the cleared status word.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ __forceinline__ float2 root_w(long long m, long long b) {  // exp(-2 pi i m / b)
+  double s, c;
+  sincospi(2.0 * (double)m / (double)b, &s, &c);
+  return make_float2((float)c, (float)(-s));
+}
+
+template <class PL>
+__global__ void setup_kernel(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed) {
+  const int tid = blockIdx.x * blockDim.x + threadIdx.x;
+  const int stride = gridDim.x * blockDim.x;
+  if (tid == 0) *status = 0u;
+  for (int e = tid; e < PL::TWN; e += stride) {
+    long long m = 0, b = 1;
+    static_for<0, PL::NP - 1>([&](auto ii) {
+      constexpr int I = decltype(ii)::value;
+      constexpr int OFF = PL::tw_off(I);
+      constexpr int LEN = PL::B(I);
+      if (e >= OFF && e < OFF + LEN) {
+        const int r = e - OFF;
+        if constexpr (I == 0) {  // [j][t]: W_N^{t j}
+          m = (long long)(r % PL::T) * (r / PL::T);
+          b = PL::N;
+        } else {                 // [j][np]: W_B^{np j}
+          constexpr int S = PL::S(I);
+          m = (long long)(r % S) * (r / S);
+          b = LEN;
+        }
+      }
+    });
+    twt[e] = root_w(m, b);
+  }
+  constexpr int words = (PL::N + 31) / 32;
+  for (int wd = tid; wd < words; wd += stride) {
+    uint32_t bits = 0;
+    for (int bb = 0; bb < 32; ++bb) {
+      const int j = wd * 32 + bb;
+      if (j >= PL::N) break;
+      const uint64_t z = splitmix64_mix(seed + (uint64_t)(j + 1) * 0x9E3779B97F4A7C15ull);
+      bits |= (uint32_t)(z >> 63) << bb;
+    }
+    eps[wd] = bits;
+  }
+}
+
+}  // namespace kd

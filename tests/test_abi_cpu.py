@@ -63,10 +63,10 @@ def test_supported_lengths(kd):
 
 
 def test_workspace_size_register_plans(kd):
-    # plans that keep u in registers need only the tables: no device query
+    # plans that keep u on chip need only the tables: no device query
     for n in (256, 768, 4096):
         ws = kd.kd_workspace_size(n)
-        assert ws >= 256 + 16 * n and ws % 256 == 0
+        assert ws >= 256 + 8 * n + n // 8 and ws % 256 == 0   # status, sign bits, pass-0 twiddles
     assert kd.kd_workspace_size(100) == 0
 
 
