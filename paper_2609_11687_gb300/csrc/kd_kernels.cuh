@@ -269,67 +269,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
     };
     auto add_none = [&](int, float, float) {};
 
-    int step = 0;
-    for (int t = 0; t < p.iters; ++t) {
-      // two greedy steps from Q_N (update u).  With u outside registers, step 1's
-      // signs are kept as bits and u is updated once after step 2 as
-      // (u + d1) + d2 -- the same roundings as two separate updates.
-      using Bits = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
-      Bits nzA = 0, ngA = 0, nzB = 0, ngB = 0;
-      float2 l1 = make_float2(0.f, 0.f);
-      auto rec1 = [&](int j, float dA, float dB) {
-        if constexpr (PL::UMODE == UREG) {
-          add_u(j, dA, dB);
-        } else {
-          nzA |= (Bits)(dA != 0.f) << j;
-          ngA |= (Bits)(dA < 0.f) << j;
-          nzB |= (Bits)(dB != 0.f) << j;
-          ngB |= (Bits)(dB < 0.f) << j;
-        }
-      };
-      auto upd2 = [&](int j, float dA, float dB) {
-        if constexpr (PL::UMODE == UREG) {
-          add_u(j, dA, dB);
-        } else {
-          const float d1A = ((nzA >> j) & 1u) ? (((ngA >> j) & 1u) ? -l1.x : l1.x) : 0.f;
-          const float d1B = ((nzB >> j) & 1u) ? (((ngB >> j) & 1u) ? -l1.y : l1.y) : 0.f;
-          float2 uj = uslot[lt + j * T];
-          uj.x = __fadd_rn(__fadd_rn(uj.x, d1A), dA);
-          uj.y = __fadd_rn(__fadd_rn(uj.y, d1B), dB);
-          uslot[lt + j * T] = uj;
-        }
-      };
-      l1 = greedy(step, t == 0, sum0, rec1);
-      ++step;
-      float2 l2 = greedy(step, false, sum0, upd2);
-      ++step;
-      // two greedy steps from P Q_N on y = P rho (update vhat implicitly)
-      xf.apply(r);
-      mask_dead(r);
-      float2 l3 = greedy(step, false, sum0, add_none);
-      ++step;
-      float2 l4 = greedy(step, false, sum0, add_none);
-      ++step;
-      xf.apply(r);
-      mask_dead(r);
-      if (t == 0) {
-        coef[0] = l1;
-        coef[1] = l2;
-        coef[2] = l3;
-        coef[3] = l4;
-      }
-    }
-
-    // ---- residual out, then vhat = P (x - u - r) ----
     const float isA = pow2f(-sA), isB = pow2f(-sB);
-    if (active && p.resid) {
-#pragma unroll
-      for (int j = 0; j < E; ++j) {
-        const int nat = nat_of<N>(lt + j * T);
-        p.resid[colA * N + nat] = __fmul_rn(r[j].x, isA);
-        if (hasB) p.resid[colB * N + nat] = __fmul_rn(r[j].y, isB);
-      }
-    }
     auto u_at = [&](int j) -> float2 {
       if constexpr (PL::UMODE == UREG) {
         return uu_reg[j];
@@ -337,23 +277,89 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         return uslot[lt + j * T];
       }
     };
-    float2 vh[E];
+
+    // Half-block hb: even = two greedy steps from Q_N (u), odd = two from P Q_N (vhat),
+    // each followed by P; the last one (hb == 2k) forms x - u - r and its P gives vhat.
+    // One call site for the transform keeps the kernel's code footprint small.
+    using Bits = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
+    int step = 0;
+    const int HB = 2 * p.iters;
+    for (int hb = 0; hb <= HB; ++hb) {
+      if (hb == HB) {
+        if (active && p.resid) {
 #pragma unroll
-    for (int j = 0; j < E; ++j) {
-      const int nat = nat_of<N>(lt + j * T);
-      const float a = __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld)), scA);
-      const float b = hasB ? __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)), scB) : 0.f;
-      const float2 uj = u_at(j);
-      vh[j] = make_float2(__fsub_rn(__fsub_rn(a, uj.x), r[j].x), __fsub_rn(__fsub_rn(b, uj.y), r[j].y));
-    }
-    if (p.iters > 0) {
-      team_sync<PL>();  // the last transform's readers of buf are done
-      xf.apply(vh);
-      mask_dead(vh);
-    } else {
+          for (int j = 0; j < E; ++j) {
+            const int nat = nat_of<N>(lt + j * T);
+            p.resid[colA * N + nat] = __fmul_rn(r[j].x, isA);
+            if (hasB) p.resid[colB * N + nat] = __fmul_rn(r[j].y, isB);
+          }
+        }
 #pragma unroll
-      for (int j = 0; j < E; ++j) vh[j] = make_float2(0.f, 0.f);
+        for (int j = 0; j < E; ++j) {
+          const int nat = nat_of<N>(lt + j * T);
+          const float a = __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld)), scA);
+          const float b =
+              hasB ? __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)), scB) : 0.f;
+          const float2 uj = u_at(j);
+          r[j] = make_float2(__fsub_rn(__fsub_rn(a, uj.x), r[j].x), __fsub_rn(__fsub_rn(b, uj.y), r[j].y));
+        }
+        if (p.iters == 0) {
+#pragma unroll
+          for (int j = 0; j < E; ++j) r[j] = make_float2(0.f, 0.f);
+          break;
+        }
+        team_sync<PL>();  // the last transform's readers of buf are done
+      } else if ((hb & 1) == 0) {
+        // two greedy steps from Q_N (update u).  With u outside registers, step 1's
+        // signs are kept as bits and u is updated once after step 2 as
+        // (u + d1) + d2 -- the same roundings as two separate updates.
+        Bits nzA = 0, ngA = 0, nzB = 0, ngB = 0;
+        float2 l1 = make_float2(0.f, 0.f);
+        auto rec1 = [&](int j, float dA, float dB) {
+          if constexpr (PL::UMODE == UREG) {
+            add_u(j, dA, dB);
+          } else {
+            nzA |= (Bits)(dA != 0.f) << j;
+            ngA |= (Bits)(dA < 0.f) << j;
+            nzB |= (Bits)(dB != 0.f) << j;
+            ngB |= (Bits)(dB < 0.f) << j;
+          }
+        };
+        auto upd2 = [&](int j, float dA, float dB) {
+          if constexpr (PL::UMODE == UREG) {
+            add_u(j, dA, dB);
+          } else {
+            const float d1A = ((nzA >> j) & 1u) ? (((ngA >> j) & 1u) ? -l1.x : l1.x) : 0.f;
+            const float d1B = ((nzB >> j) & 1u) ? (((ngB >> j) & 1u) ? -l1.y : l1.y) : 0.f;
+            float2 uj = uslot[lt + j * T];
+            uj.x = __fadd_rn(__fadd_rn(uj.x, d1A), dA);
+            uj.y = __fadd_rn(__fadd_rn(uj.y, d1B), dB);
+            uslot[lt + j * T] = uj;
+          }
+        };
+        l1 = greedy(step, hb == 0, sum0, rec1);
+        ++step;
+        const float2 l2 = greedy(step, false, sum0, upd2);
+        ++step;
+        if (hb == 0) {
+          coef[0] = l1;
+          coef[1] = l2;
+        }
+      } else {
+        // two greedy steps from P Q_N on y = P rho (vhat is implicit: P (x - u - r) at the end)
+        const float2 l3 = greedy(step, false, sum0, add_none);
+        ++step;
+        const float2 l4 = greedy(step, false, sum0, add_none);
+        ++step;
+        if (hb == 1) {
+          coef[2] = l3;
+          coef[3] = l4;
+        }
+      }
+      xf.apply(r);
+      mask_dead(r);
     }
+    float2(&vh)[E] = r;  // r now holds vhat
 
     // ---- optional dense factors (natural order, scaled back) ----
     if (active && (p.u || p.vhat)) {

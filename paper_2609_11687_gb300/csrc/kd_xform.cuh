@@ -45,7 +45,7 @@ struct Plan {
   static constexpr int RL = Rv[NP - 1];
   static constexpr int THREADS = T * Q;
   static constexpr int NW = (T + 31) / 32;  // warps per team
-  static constexpr int BUF = (N + N / 16 + 8 + 15) / 16 * 16;  // padded float2 slots per team
+  static constexpr int BUF = (N + N / 16 + N / 256 + 8 + 15) / 16 * 16;  // padded float2 slots per team
   static constexpr int RED = 4 * (NW > 1 ? NW : 1);           // float2 reduction slots per team
   static constexpr int USL = (UMODE_ == 2) ? N : 0;            // float2 slots of u per team (shared)
   // M in registers: one last-pass group per thread, partner at lane ^ HALF
@@ -85,7 +85,9 @@ struct Plan {
   static_assert(valid(), "inconsistent plan");
 };
 
-__device__ __forceinline__ int pad(int i) { return i + (i >> 4); }
+// Padded slot: one spare float2 per 16 and per 256 slots, so that accesses with
+// lane strides 1, 16 and 256 fall in distinct bank pairs.
+__device__ __forceinline__ int pad(int i) { return i + (i >> 4) + (i >> 8); }
 
 // Twiddle read that the compiler may not hoist out of the block loop: every
 // thread's twiddles are loop-invariant, and keeping them all in registers would
