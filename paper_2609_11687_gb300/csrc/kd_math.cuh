@@ -69,11 +69,13 @@ KD_HD constexpr double sin2pi(long long a, long long b) {
 // ---------------------------------------------------------------------------
 // Complex helpers (float2 = re, im)
 // ---------------------------------------------------------------------------
+// Complex add / subtract as one packed FP32x2 fused multiply-add with +-1 (the
+// same rounding as separate adds: b * 1 is exact), half the issue slots.
 __device__ __forceinline__ float2 cadd(float2 a, float2 b) {
-  return make_float2(__fadd_rn(a.x, b.x), __fadd_rn(a.y, b.y));
+  return __ffma2_rn(b, make_float2(1.f, 1.f), a);
 }
 __device__ __forceinline__ float2 csub(float2 a, float2 b) {
-  return make_float2(__fsub_rn(a.x, b.x), __fsub_rn(a.y, b.y));
+  return __ffma2_rn(b, make_float2(-1.f, -1.f), a);
 }
 // a * b
 __device__ __forceinline__ float2 cmul(float2 a, float2 b) {
@@ -236,16 +238,16 @@ template <int R, int DIR, class Load, class Store>
 __device__ __forceinline__ void dft_prime_stream(Load&& load, Store&& store) {
   constexpr int H = (R - 1) / 2;
   float2 a[H + 1], b[H + 1];
-  const float2 x0 = load(0);
+  const float2 x0 = load(ic<0>{});
   float2 sum = x0;
-#pragma unroll
-  for (int n = 1; n <= H; ++n) {
-    const float2 p = load(n), q = load(R - n);
-    a[n] = cadd(p, q);
-    b[n] = csub(p, q);
-    sum = cadd(sum, a[n]);
-  }
-  store(0, sum);
+  static_for<1, H + 1>([&](auto nc) {
+    constexpr int NN = decltype(nc)::value;
+    const float2 p = load(ic<NN>{}), q = load(ic<R - NN>{});
+    a[NN] = cadd(p, q);
+    b[NN] = csub(p, q);
+    sum = cadd(sum, a[NN]);
+  });
+  store(ic<0>{}, sum);
   static_for<1, H + 1>([&](auto kk) {
     constexpr int K = decltype(kk)::value;
     float2 ak = x0;
@@ -261,11 +263,11 @@ __device__ __forceinline__ void dft_prime_stream(Load&& load, Store&& store) {
     });
     const float2 ib = mul_pi(bk);
     if constexpr (DIR < 0) {
-      store(K, csub(ak, ib));
-      store(R - K, cadd(ak, ib));
+      store(ic<K>{}, csub(ak, ib));
+      store(ic<R - K>{}, cadd(ak, ib));
     } else {
-      store(K, cadd(ak, ib));
-      store(R - K, csub(ak, ib));
+      store(ic<K>{}, cadd(ak, ib));
+      store(ic<R - K>{}, csub(ak, ib));
     }
   });
 }

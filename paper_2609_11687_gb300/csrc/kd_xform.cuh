@@ -32,6 +32,41 @@ namespace kd {
 
 enum { UREG = 0, UGMEM = 1, USMEM = 2 };
 
+// Padded slot: one spare float2 per 16 and per 256 slots, so that accesses with
+// lane strides 1, 16 and 256 fall in distinct bank pairs.
+KD_HD constexpr int pad(int i) { return i + (i >> 4) + (i >> 8); }
+
+// True when pad(base + j*stride) == pad(base) + pad(j*stride) for every base the
+// access pattern produces (checked exhaustively at compile time), so element
+// addresses are a per-thread padded base plus compile-time offsets.
+KD_HD constexpr bool sep_strided(int nbase, int base_mul, int base_add_max, int count, int stride) {
+  // bases: b = q * base_mul + a, q < nbase, a < base_add_max
+  for (int q = 0; q < nbase; ++q)
+    for (int a = 0; a < base_add_max; ++a) {
+      const int b = q * base_mul + a;
+      for (int j = 0; j < count; ++j)
+        if (pad(b + j * stride) != pad(b) + pad(j * stride)) return false;
+    }
+  return true;
+}
+
+// Twiddle read that the compiler may not hoist out of the block loop: every
+// thread's twiddles are loop-invariant, and keeping them all in registers would
+// spill.  SMEM selects a shared-memory (else read-only global) load.
+template <bool SMEM>
+__device__ __forceinline__ float2 ld_tw(const float2* p) {
+  float2 v;
+  if constexpr (SMEM) {
+    const unsigned a = (unsigned)__cvta_generic_to_shared(p);
+    asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
+  } else {
+    asm volatile("ld.global.nc.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(p));
+  }
+  return v;
+}
+
+
+
 template <int N_, int T_, int Q_, int UMODE_, int MINB_, int... Rs>
 struct Plan {
   static constexpr int N = N_;
@@ -76,6 +111,27 @@ struct Plan {
   static constexpr size_t SMEM_TW = TW_SMEM ? (size_t)TWN * sizeof(float2) : 0;
   static constexpr size_t SMEM = SMEM_TW + (size_t)Q * TEAM * sizeof(float2);
 
+  // pass 0 / inverse pass 0 and slot-order M: slots base + j*T with base < T
+  static constexpr bool SEP0 = sep_strided(1, 0, T, E, T);
+  // paired last pass: group of frequencies K + (N/RL) j sits at slot_low(K) + j
+  KD_HD static constexpr int slot_low_c(int K) {
+    int s = 0;
+    for (int i = 0; i < NP - 1; ++i) {
+      s += (K % Rv[i]) * (B(i) / Rv[i]);
+      K /= Rv[i];
+    }
+    return s;
+  }
+  KD_HD static constexpr bool sep_last() {
+    for (int K = 0; K < N / RL; ++K)
+      for (int j = 0; j < RL; ++j)
+        if (pad(slot_low_c(K) + j) != pad(slot_low_c(K)) + pad(j)) return false;
+    return true;
+  }
+  KD_HD static constexpr bool sep_pass(int i) {
+    // groups of pass i: base = blk * B(i) + np (blk < N/B(i), np < S(i)), stride S(i)
+    return sep_strided(N / B(i), B(i), S(i), Rv[i], S(i));
+  }
   KD_HD static constexpr bool valid() {
     int p = 1;
     for (int i = 0; i < NP; ++i) p *= Rv[i];
@@ -84,25 +140,6 @@ struct Plan {
   }
   static_assert(valid(), "inconsistent plan");
 };
-
-// Padded slot: one spare float2 per 16 and per 256 slots, so that accesses with
-// lane strides 1, 16 and 256 fall in distinct bank pairs.
-__device__ __forceinline__ int pad(int i) { return i + (i >> 4) + (i >> 8); }
-
-// Twiddle read that the compiler may not hoist out of the block loop: every
-// thread's twiddles are loop-invariant, and keeping them all in registers would
-// spill.  SMEM selects a shared-memory (else read-only global) load.
-template <bool SMEM>
-__device__ __forceinline__ float2 ld_tw(const float2* p) {
-  float2 v;
-  if constexpr (SMEM) {
-    const unsigned a = (unsigned)__cvta_generic_to_shared(p);
-    asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
-  } else {
-    asm volatile("ld.global.nc.v2.f32 {%0, %1}, [%2];" : "=f"(v.x), "=f"(v.y) : "l"(p));
-  }
-  return v;
-}
 
 template <class PL>
 __device__ __forceinline__ void team_sync() {
@@ -175,6 +212,8 @@ struct Xform {
   using Mask = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
   Mask ek, em;                 // eps_k < 0 / eps_{-k} < 0 for each owned frequency (bit index)
   int p0, p1;                  // slot-order M: partner slot constants
+  int pb0;                     // pad(lt): base of the pass-0 slots lt + j T
+  int pbp0, pbp1;              // slot-order M: pad(p0), pad(p1)
   int kgrp;                    // paired M: own frequency group (k = kgrp + (N/RL) j)
   int lbase;                   // paired M: slot of that group's first element
   int self;                    // paired M: 0 regular, 1 group 0, 2 group N/(2 R0)
@@ -183,6 +222,7 @@ struct Xform {
     buf = b;
     tw = t;
     lt = lane_t;
+    pb0 = pad(lt);
     ek = em = 0;
     if constexpr (PL::PAIRED) {
       constexpr int H = PL::HALF;
@@ -199,11 +239,13 @@ struct Xform {
         ek |= (Mask)eps_neg(eb, k) << kp;
         em |= (Mask)eps_neg(eb, (N - k) % N) << kp;
       }
-      p0 = p1 = 0;
+      p0 = p1 = pbp0 = pbp1 = 0;
     } else {
       const int Kp = rest_of_slot<PL>(lt);
       p0 = slot_rest<PL>((T - Kp) % T);
       p1 = slot_rest<PL>(T - 1 - Kp);
+      pbp0 = pad(p0);
+      pbp1 = pad(p1);
       cw = expi_pi((long long)E * Kp, N);
 #pragma unroll
       for (int r = 0; r < E; ++r) {
@@ -213,6 +255,13 @@ struct Xform {
       }
       kgrp = self = lbase = 0;
     }
+  }
+
+  // padded address of pass-0 slot lt + j T (base + compile-time offset when separable)
+  template <int J>
+  __device__ __forceinline__ int a0() const {
+    if constexpr (PL::SEP0) return pb0 + pad(J * T);
+    else return pad(lt + J * T);
   }
 
   // M on one frequency: own value a, partner value b; returns Z'_k (1/N folded in).
@@ -232,19 +281,20 @@ struct Xform {
   // forward pass 0 from registers
   __device__ __forceinline__ void fwd0(float2 (&v)[E]) {
     if constexpr (kd_is_big_prime<E>()) {
-      dft_prime_stream<E, -1>([&](int j) { return v[j]; },
-                              [&](int k, float2 x) {
-                                if (k > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + k * T + lt));
-                                buf[pad(lt + k * T)] = x;
+      dft_prime_stream<E, -1>([&](auto jc) { return v[decltype(jc)::value]; },
+                              [&](auto kc, float2 x) {
+                                constexpr int K = decltype(kc)::value;
+                                if constexpr (K > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + K * T + lt));
+                                buf[a0<K>()] = x;
                               });
     } else {
       Dft<E, -1>::run(v);
-#pragma unroll
-      for (int j = 0; j < E; ++j) {
-        float2 x = v[j];
-        if (j > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + j * T + lt));
-        buf[pad(lt + j * T)] = x;
-      }
+      static_for<0, E>([&](auto jc) {
+        constexpr int J = decltype(jc)::value;
+        float2 x = v[J];
+        if constexpr (J > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));
+        buf[a0<J>()] = x;
+      });
     }
   }
 
@@ -253,21 +303,21 @@ struct Xform {
     if constexpr (kd_is_big_prime<E>()) {
       // outputs go back to the thread's own slots (already read), then to registers
       dft_prime_stream<E, +1>(
-          [&](int j) {
-            float2 x = buf[pad(lt + j * T)];
-            if (j > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + j * T + lt));
+          [&](auto jc) {
+            constexpr int J = decltype(jc)::value;
+            float2 x = buf[a0<J>()];
+            if constexpr (J > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));
             return x;
           },
-          [&](int k, float2 x) { buf[pad(lt + k * T)] = x; });
-#pragma unroll
-      for (int j = 0; j < E; ++j) v[j] = buf[pad(lt + j * T)];
+          [&](auto kc, float2 x) { buf[a0<decltype(kc)::value>()] = x; });
+      static_for<0, E>([&](auto jc) { v[decltype(jc)::value] = buf[a0<decltype(jc)::value>()]; });
     } else {
-#pragma unroll
-      for (int j = 0; j < E; ++j) {
-        float2 x = buf[pad(lt + j * T)];
-        if (j > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + j * T + lt));
-        v[j] = x;
-      }
+      static_for<0, E>([&](auto jc) {
+        constexpr int J = decltype(jc)::value;
+        float2 x = buf[a0<J>()];
+        if constexpr (J > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));
+        v[J] = x;
+      });
       Dft<E, +1>::run(v);
     }
   }
@@ -281,13 +331,16 @@ struct Xform {
     constexpr int G = N / R;
     constexpr bool LAST = (I == NP - 1);
     constexpr int OFF = PL::tw_off(I);
+    constexpr bool SEP = PL::sep_pass(I);
     for (int g = lt; g < G; g += T) {
       const int blk = g / S;
       const int np = g - blk * S;
       const int base = blk * Bk + np;
+      const int pb = pad(base);
+      auto addr = [&](int j) { return SEP ? pb + pad(j * S) : pad(base + j * S); };
       float2 v[R];
 #pragma unroll
-      for (int j = 0; j < R; ++j) v[j] = buf[pad(base + j * S)];
+      for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
       if constexpr (DIR < 0) {
         Dft<R, -1>::run(v);
         if constexpr (!LAST) {
@@ -302,7 +355,7 @@ struct Xform {
         Dft<R, +1>::run(v);
       }
 #pragma unroll
-      for (int j = 0; j < R; ++j) buf[pad(base + j * S)] = v[j];
+      for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
     }
   }
 
@@ -310,10 +363,13 @@ struct Xform {
   __device__ __forceinline__ void last_paired() {
     constexpr int R = PL::RL;
     constexpr int H = PL::HALF;
+    constexpr bool SEP = PL::sep_last();
     const int base = lbase;
+    const int pb = pad(base);
+    auto addr = [&](int j) { return SEP ? pb + pad(j) : pad(base + j); };
     float2 v[R];
 #pragma unroll
-    for (int j = 0; j < R; ++j) v[j] = buf[pad(base + j)];
+    for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
     Dft<R, -1>::run(v);
     float2 o[R];
     static_for<0, R>([&](auto kk) {
@@ -329,21 +385,22 @@ struct Xform {
     });
     Dft<R, +1>::run(o);
 #pragma unroll
-    for (int j = 0; j < R; ++j) buf[pad(base + j)] = o[j];
+    for (int j = 0; j < R; ++j) buf[addr(j)] = o[j];
   }
 
   // slot-order M (own slots lt + T r, partners from constants); v is scratch
   __device__ __forceinline__ void middle_slots(float2 (&v)[E]) {
     static_for<0, E>([&](auto rr) {
       constexpr int RR = decltype(rr)::value;
-      const int s = lt + T * RR;
-      const int ps = (RR == 0) ? p0 : (E - RR) * T + p1;
+      int pa;
+      if constexpr (RR == 0) pa = pbp0;
+      else if constexpr (PL::SEP0) pa = pbp1 + pad((E - RR) * T);
+      else pa = pad((E - RR) * T + p1);
       // k = RR + E K': exp(i pi k/N) = exp(i pi E K'/N) exp(i pi RR/N)
-      v[RR] = mfreq<RR, N>(buf[pad(s)], buf[pad(ps)], RR);
+      v[RR] = mfreq<RR, N>(buf[a0<RR>()], buf[pa], RR);
     });
     team_sync<PL>();
-#pragma unroll
-    for (int r = 0; r < E; ++r) buf[pad(lt + T * r)] = v[r];
+    static_for<0, E>([&](auto rr) { buf[a0<decltype(rr)::value>()] = v[decltype(rr)::value]; });
   }
 
   // y = P' v
