@@ -179,7 +179,8 @@ def run_gpu(args) -> dict:
     dev = torch.device("cuda", local)
     # this rank's layers: rank, rank + world, ...  (weak scaling, no data exchange)
     steps_total = args.warmup + args.steps
-    my_layers = [(rank + world * i) % LAYERS for i in range(steps_total)]
+    from paper_2609_11687_gb300 import shard
+    my_layers = shard.layer_schedule(rank, world, steps_total, LAYERS)
     uniq = sorted(set(my_layers))
     log(f"[bench] rank {rank}/{world}: generating {len(uniq)} Llama-2-7B-shaped layers on {dev}")
     t0 = time.time()
@@ -243,12 +244,8 @@ def run_gpu(args) -> dict:
     if dist:
         dist.barrier()
     clk = clocks.stop()
-    elapsed_ms = start.elapsed_time(end)
-    t = torch.tensor([elapsed_ms], device=dev)
-    if dist:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    elapsed_ms = float(t.item())
-    value = world * args.steps * layer_params / (elapsed_ms / 1e3)
+    elapsed_ms, total_params = shard.aggregate(start.elapsed_time(end), args.steps * layer_params)
+    value = total_params / (elapsed_ms / 1e3)
 
     # dominant kernel: average launch duration over the timed region
     launches = ev_main.get("ev", [])
@@ -337,13 +334,10 @@ def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
         step()
     b.record(stream)
     torch.cuda.synchronize()
-    ms = a.elapsed_time(b)
-    t = torch.tensor([ms], device=stream.device)
-    if dist:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms = float(t.item())
+    from paper_2609_11687_gb300 import shard
     params = sum(s.params for s, _ in layer)
-    return {"value": round(world * n * params / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
+    ms, total = shard.aggregate(a.elapsed_time(b), n * params)
+    return {"value": round(total / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": n}
 
 
