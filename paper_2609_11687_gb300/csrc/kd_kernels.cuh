@@ -320,17 +320,17 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
             add_u(j, dA, dB);
           } else {
             nzA |= (Bits)(dA != 0.f) << j;
-            ngA |= (Bits)(dA < 0.f) << j;
+            ngA |= (Bits)(__float_as_uint(dA) >> 31) << j;
             nzB |= (Bits)(dB != 0.f) << j;
-            ngB |= (Bits)(dB < 0.f) << j;
+            ngB |= (Bits)(__float_as_uint(dB) >> 31) << j;
           }
         };
         auto upd2 = [&](int j, float dA, float dB) {
           if constexpr (PL::UMODE == UREG) {
             add_u(j, dA, dB);
           } else {
-            const float d1A = ((nzA >> j) & 1u) ? (((ngA >> j) & 1u) ? -l1.x : l1.x) : 0.f;
-            const float d1B = ((nzB >> j) & 1u) ? (((ngB >> j) & 1u) ? -l1.y : l1.y) : 0.f;
+            const float d1A = ((nzA >> j) & 1u) ? __uint_as_float(__float_as_uint(l1.x) | (uint32_t)((ngA >> j) & 1u) << 31) : 0.f;
+            const float d1B = ((nzB >> j) & 1u) ? __uint_as_float(__float_as_uint(l1.y) | (uint32_t)((ngB >> j) & 1u) << 31) : 0.f;
             float2 uj = uslot[lt + j * T];
             uj.x = __fadd_rn(__fadd_rn(uj.x, d1A), dA);
             uj.y = __fadd_rn(__fadd_rn(uj.y, d1B), dB);

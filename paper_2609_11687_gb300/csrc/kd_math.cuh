@@ -94,6 +94,14 @@ __device__ __forceinline__ float2 cscale(float2 a, float s) {
 __device__ __forceinline__ float2 mul_mi(float2 a) { return make_float2(a.y, -a.x); }
 // +i * a   (exact)
 __device__ __forceinline__ float2 mul_pi(float2 a) { return make_float2(-a.y, a.x); }
+// a + i b and a - i b as two scalar adds: the swapped operand would need register
+// moves in packed form.
+__device__ __forceinline__ float2 add_ib(float2 a, float2 b) {
+  return make_float2(__fsub_rn(a.x, b.y), __fadd_rn(a.y, b.x));
+}
+__device__ __forceinline__ float2 sub_ib(float2 a, float2 b) {
+  return make_float2(__fadd_rn(a.x, b.y), __fsub_rn(a.y, b.x));
+}
 
 // Multiply by the compile-time root W_R^E = exp(DIR * 2 pi i E / R), DIR = -1 forward.
 // Quarter turns are exact; eighth turns use one constant; others a full product.
@@ -179,11 +187,15 @@ struct Dft<4, DIR> {
     float2 s02 = cadd(v[0], v[2]), d02 = csub(v[0], v[2]);
     float2 s13 = cadd(v[1], v[3]), d13 = csub(v[1], v[3]);
     // forward: X1 = d02 - i d13, X3 = d02 + i d13 ; inverse: signs swapped
-    float2 t = (DIR < 0) ? mul_mi(d13) : mul_pi(d13);
     v[0] = cadd(s02, s13);
     v[2] = csub(s02, s13);
-    v[1] = cadd(d02, t);
-    v[3] = csub(d02, t);
+    if constexpr (DIR < 0) {
+      v[1] = sub_ib(d02, d13);
+      v[3] = add_ib(d02, d13);
+    } else {
+      v[1] = add_ib(d02, d13);
+      v[3] = sub_ib(d02, d13);
+    }
   }
 };
 
@@ -218,13 +230,12 @@ struct DftPrime {
         bk.y = __fmaf_rn(b[NN].y, s, bk.y);
       });
       // forward: X_k = ak - i bk, X_{R-k} = ak + i bk ; inverse: the reverse
-      const float2 ib = mul_pi(bk);
       if constexpr (DIR < 0) {
-        v[K] = csub(ak, ib);
-        v[R - K] = cadd(ak, ib);
+        v[K] = sub_ib(ak, bk);
+        v[R - K] = add_ib(ak, bk);
       } else {
-        v[K] = cadd(ak, ib);
-        v[R - K] = csub(ak, ib);
+        v[K] = add_ib(ak, bk);
+        v[R - K] = sub_ib(ak, bk);
       }
     });
   }
@@ -261,13 +272,12 @@ __device__ __forceinline__ void dft_prime_stream(Load&& load, Store&& store) {
       bk.x = __fmaf_rn(b[NN].x, sn, bk.x);
       bk.y = __fmaf_rn(b[NN].y, sn, bk.y);
     });
-    const float2 ib = mul_pi(bk);
     if constexpr (DIR < 0) {
-      store(ic<K>{}, csub(ak, ib));
-      store(ic<R - K>{}, cadd(ak, ib));
+      store(ic<K>{}, sub_ib(ak, bk));
+      store(ic<R - K>{}, add_ib(ak, bk));
     } else {
-      store(ic<K>{}, cadd(ak, ib));
-      store(ic<R - K>{}, csub(ak, ib));
+      store(ic<K>{}, add_ib(ak, bk));
+      store(ic<R - K>{}, sub_ib(ak, bk));
     }
   });
 }

@@ -26,6 +26,8 @@
 // a few per-thread constants computed once per CTA.
 #pragma once
 
+#include <type_traits>
+
 #include "kd_math.cuh"
 
 namespace kd {
@@ -211,6 +213,8 @@ struct Xform {
   float2 cw;                   // M twiddle base
   using Mask = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
   Mask ek, em;                 // eps_k < 0 / eps_{-k} < 0 for each owned frequency (bit index)
+  Mask dm;                     // ek ^ em: frequencies whose M takes the partner value
+  static constexpr float kInvN = 1.0f / (float)N;
   int p0, p1;                  // slot-order M: partner slot constants
   int pb0;                     // pad(lt): base of the pass-0 slots lt + j T
   int pbp0, pbp1;              // slot-order M: pad(p0), pad(p1)
@@ -240,6 +244,7 @@ struct Xform {
         em |= (Mask)eps_neg(eb, (N - k) % N) << kp;
       }
       p0 = p1 = pbp0 = pbp1 = 0;
+      dm = ek ^ em;
     } else {
       const int Kp = rest_of_slot<PL>(lt);
       p0 = slot_rest<PL>((T - Kp) % T);
@@ -254,6 +259,7 @@ struct Xform {
         em |= (Mask)eps_neg(eb, (N - k) % N) << r;
       }
       kgrp = self = lbase = 0;
+      dm = ek ^ em;
     }
   }
 
@@ -265,17 +271,18 @@ struct Xform {
   }
 
   // M on one frequency: own value a, partner value b; returns Z'_k (1/N folded in).
-  template <long long RNUM, long long RDEN>
-  __device__ __forceinline__ float2 mfreq(float2 a, float2 b, int bit) const {
-    constexpr float invN = 1.0f / (float)N;
-    const bool neg = (ek >> bit) & 1u;
-    const bool negm = (em >> bit) & 1u;
-    const float f = neg ? -invN : invN;
+  // eps_k == eps_{N-k}: Z'_k = eps_k a / N;  otherwise Z'_k = eps_k exp(i pi k/N) b / N.
+  template <long long RNUM, long long RDEN, int BIT>
+  __device__ __forceinline__ float2 mfreq(float2 a, float2 b) const {
     // exp(i pi k / N) = cw * exp(i pi RNUM / RDEN)
     const float2 wk = mul_root<+1, RNUM, 2 * RDEN>(cw);
     const float2 t = cmul(b, wk);
-    const float2 sel = (neg == negm) ? a : t;
-    return cscale(sel, f);
+    const bool diff = (dm >> BIT) & 1u;
+    const float2 sel = diff ? t : a;
+    // +-1/N with the sign of eps_k taken straight from its bit
+    const uint32_t sgn = (uint32_t)((ek >> BIT) & 1u) << 31;
+    const float f = __uint_as_float(__float_as_uint(kInvN) | sgn);
+    return __fmul2_rn(sel, make_float2(f, f));
   }
 
   // forward pass 0 from registers
@@ -372,17 +379,29 @@ struct Xform {
     for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
     Dft<R, -1>::run(v);
     float2 o[R];
-    static_for<0, R>([&](auto kk) {
-      constexpr int KP = decltype(kk)::value;
-      const float2 src = v[R - 1 - KP];
-      float2 q;
-      q.x = __shfl_xor_sync(0xffffffffu, src.x, H);
-      q.y = __shfl_xor_sync(0xffffffffu, src.y, H);
-      if (self == 1) q = v[(R - KP) % R];
-      else if (self == 2) q = v[R - 1 - KP];
-      // k = K + (N/R) KP: exp(i pi k/N) = exp(i pi K/N) exp(i pi KP/R)
-      o[KP] = mfreq<KP, R>(v[KP], q, KP);
-    });
+    // Only the warp holding groups 0 and N/(2 RL) (self-paired) needs the local-value
+    // selects; every other warp takes the shuffle-only path (warp-uniform branch).
+    auto body = [&](auto slowc) {
+      constexpr bool SLOW = decltype(slowc)::value;
+      static_for<0, R>([&](auto kk) {
+        constexpr int KP = decltype(kk)::value;
+        const float2 src = v[R - 1 - KP];
+        float2 q;
+        q.x = __shfl_xor_sync(0xffffffffu, src.x, H);
+        q.y = __shfl_xor_sync(0xffffffffu, src.y, H);
+        if constexpr (SLOW) {
+          if (self == 1) q = v[(R - KP) % R];
+          else if (self == 2) q = src;
+        }
+        // k = K + (N/R) KP: exp(i pi k/N) = exp(i pi K/N) exp(i pi KP/R)
+        o[KP] = mfreq<KP, R, KP>(v[KP], q);
+      });
+    };
+    if (__any_sync(0xffffffffu, self != 0)) {
+      body(std::true_type{});
+    } else {
+      body(std::false_type{});
+    }
     Dft<R, +1>::run(o);
 #pragma unroll
     for (int j = 0; j < R; ++j) buf[addr(j)] = o[j];
@@ -397,7 +416,7 @@ struct Xform {
       else if constexpr (PL::SEP0) pa = pbp1 + pad((E - RR) * T);
       else pa = pad((E - RR) * T + p1);
       // k = RR + E K': exp(i pi k/N) = exp(i pi E K'/N) exp(i pi RR/N)
-      v[RR] = mfreq<RR, N>(buf[a0<RR>()], buf[pa], RR);
+      v[RR] = mfreq<RR, N, RR>(buf[a0<RR>()], buf[pa]);
     });
     team_sync<PL>();
     static_for<0, E>([&](auto rr) { buf[a0<decltype(rr)::value>()] = v[decltype(rr)::value]; });
