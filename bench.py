@@ -118,7 +118,7 @@ class ClockSampler:
 # CPU oracle baseline (bounded sample)
 # ---------------------------------------------------------------------------
 
-def oracle_baseline(specs, iters: int, budget_s: float = 12.0) -> dict:
+def oracle_baseline(specs, iters: int, budget_s: float = 12.0, kmeans_iters: int = 0) -> dict:
     """Time the CPU oracle as it stands on a bounded sample of the layer and scale
     to params/s of the whole layer mix (time per parameter measured per vector
     length, weighted by the layer's parameters at that length)."""
@@ -135,25 +135,33 @@ def oracle_baseline(specs, iters: int, budget_s: float = 12.0) -> dict:
         spec = group[0]
         import torch
         import dataclasses
-        G = synth.generate(dataclasses.replace(spec, M=64))
+        G = synth.generate(dataclasses.replace(spec, M=512))
         x = G.double().numpy().T
         eps = ko.sign_mask(spec.sign_seed, n)
         P = ko.POperator(n, eps)
         m = 2
         while True:
             t0 = time.perf_counter()
-            ko.decompose(x[:, :m], eps, iters, P=P)
+            d = ko.decompose(x[:, :m], eps, iters, P=P)
+            cu = ko.centres(d.coeffs[0], d.coeffs[1])
+            cv = ko.centres(d.coeffs[2], d.coeffs[3])
+            if kmeans_iters:
+                cu, code_u, _, _ = ko.kmeans_refine(d.u, cu, kmeans_iters)
+                cv, code_v, _, _ = ko.kmeans_refine(d.vhat, cv, kmeans_iters)
+            else:
+                code_u, code_v = ko.codes(d.u, cu), ko.codes(d.vhat, cv)
+            ko.pack_codes(code_u), ko.pack_codes(code_v)
             dt = time.perf_counter() - t0
-            if dt > share / 4 or m >= 64:
+            if dt > share / 4 or m >= 512:
                 break
-            m = min(64, m * 2)
+            m = min(512, m * 2)
         per_param[n] = dt / (m * n)
         sample_desc.append(f"{m} vectors of n={n} ({dt:.1f}s)")
     layer_params = sum(s.params for s in specs)
     layer_time = sum(s.params * per_param[s.N] for s in specs)
     return {"value": layer_params / layer_time, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
-            "sample": "fp64 dense-DCT oracle, k=%d, on %s, scaled to the layer's parameter mix (seeded "
-                      "Student-t vectors of the layer's shapes)" % (iters, "; ".join(sample_desc))}
+            "sample": "fp64 dense-DCT oracle, k=%d, kmeans=%d, on %s, scaled to the layer's parameter mix (seeded "
+                      "Student-t vectors of the layer's shapes)" % (iters, kmeans_iters, "; ".join(sample_desc))}
 
 
 # ---------------------------------------------------------------------------
@@ -218,7 +226,8 @@ def run_gpu(args) -> dict:
                 e0 = torch.cuda.Event(enable_timing=True)
                 e1 = torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-            kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream)
+            kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream,
+                         kmeans_iters=args.kmeans_iters)
             if record and s.N == 4096:
                 e1.record(stream)
                 ev_main.setdefault("ev", []).append((e0, e1, s.M))
@@ -267,6 +276,12 @@ def run_gpu(args) -> dict:
     if clk.get("sm_mhz"):
         roofline["frac_at_measured_clock"] = round(achieved_tflops / (peak * clk["sm_mhz"] / 2070.0), 4)
 
+    # k-means refinement (Sec. 2.1): cost of KM_PROBE Lloyd iterations on the dominant
+    # kernel, timed on the same matrices right after the timed region
+    refinement = None
+    if args.kmeans_iters == 0:
+        refinement = measure_refinement(kd, torch, layers[my_layers[-1]], outs, wss, iters, stream, dur)
+
     # end to end: pinned host input, H2D + decompose + D2H codes/centres each step
     e2e = None
     if not args.skip_e2e:
@@ -279,20 +294,49 @@ def run_gpu(args) -> dict:
         "config": {"workload": "llama2-7b decoder layer per step: q,k,v,o 4096x4096, gate,up 4096x11008, "
                                "down 11008x4096 (202,375,168 params, fp16 Student-t nu=4 std 0.015, 0.1% input "
                                "channels x20), cycling the 32 seeded layers of the 7B stack resident in HBM",
-                   "iters": iters, "layout": "vector-major (nn.Linear [out, in])",
+                   "iters": iters, "kmeans_iters": args.kmeans_iters,
+                   "layout": "vector-major (nn.Linear [out, in])",
                    "l2": "inputs larger than L2 (405 MB per step, distinct layer every step)",
                    "parallelism": f"dp{world} (layers sharded over ranks, no exchange)"},
         "roofline": roofline,
         "gpu_launches": args.steps * 7 * 2,
         "clocks": clk,
     }
+    if refinement is not None:
+        result["kmeans_refinement"] = refinement
     if e2e is not None:
         result["e2e"] = e2e
     if rank == 0 and world == 1 and not args.skip_cpu:
-        result["cpu_baseline"] = oracle_baseline(synth.llama7b_layer(0), iters, budget_s=args.cpu_budget)
+        result["cpu_baseline"] = oracle_baseline(synth.llama7b_layer(0), iters, budget_s=args.cpu_budget,
+                                                 kmeans_iters=args.kmeans_iters)
     if dist:
         dist.destroy_process_group()
     return result if rank == 0 else None
+
+
+KM_PROBE = 3
+
+
+def measure_refinement(kd, torch, layer, outs, wss, iters, stream, base_ms):
+    """Average N = 4096 launch time with KM_PROBE refinement iterations, against the
+    closed-form launch time measured in the timed region."""
+    evs = []
+    for rep in range(3):
+        for s, w in layer:
+            if s.N != 4096:
+                continue
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=outs[(s.N, s.M)], stream=stream,
+                         kmeans_iters=KM_PROBE)
+            b.record(stream)
+            if rep > 0:
+                evs.append((a, b))
+    torch.cuda.synchronize()
+    ms = sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+    return {"kmeans_iters": KM_PROBE, "kernel": "decompose_kernel<N=4096>", "launch_ms": round(ms, 3),
+            "overhead_vs_closed_form": round(ms / base_ms - 1.0, 4)}
 
 
 def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
@@ -314,7 +358,8 @@ def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
         for (s, hw), dw in zip(host_in, dev_in):
             dw.copy_(hw, non_blocking=True)
             o = outs[(s.N, s.M)]
-            kd.decompose(dw, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream)
+            kd.decompose(dw, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream,
+                         kmeans_iters=args.kmeans_iters)
             hu, hv, hcu, hcv = host_out[(s.N, s.M)]
             hu.copy_(o.codes_u, non_blocking=True)
             hv.copy_(o.codes_v, non_blocking=True)
@@ -354,7 +399,7 @@ def run_reference(args) -> dict | None:
     budget = max(2.0, min(30.0, 150.0 / max(1, args.steps + args.warmup)))
     vals = []
     for i in range(args.warmup + args.steps):
-        b = oracle_baseline(specs, args.iters, budget_s=budget)
+        b = oracle_baseline(specs, args.iters, budget_s=budget, kmeans_iters=args.kmeans_iters)
         if i >= args.warmup:
             vals.append(b)
     value = sum(v["value"] for v in vals) / len(vals)
@@ -365,7 +410,8 @@ def run_reference(args) -> dict | None:
         "ms_per_step": layer_params / value * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": "llama2-7b decoder layer per step (202,375,168 params), each timed step a "
-                               "bounded sample of that layer on the host cores", "iters": args.iters},
+                               "bounded sample of that layer on the host cores", "iters": args.iters,
+                   "kmeans_iters": args.kmeans_iters},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                          "sample": vals[-1]["sample"]},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -396,6 +442,8 @@ def main():
     ap.add_argument("--steps", type=int, default=32)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--iters", type=int, default=ITERS)
+    ap.add_argument("--kmeans-iters", type=int, default=0,
+                    help="Lloyd refinement iterations of the centres (Sec. 2.1); 0 = closed form")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")

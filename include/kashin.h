@@ -87,23 +87,31 @@ kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host);
  *  w          input, dtype elements, `layout` with leading dimension ld.
  *  iters      k >= 0 blocks of four atomic greedy steps (two on Q_N -> u, two on
  *             P Q_N -> vhat).  k = 0 gives zero factors, zero centres, codes 0.
+ *  kmeans_iters  0..64 Lloyd refinement iterations of each factor's 4 centres from
+ *             the closed form (Sec. 2.1: "a small number of k-means refinement
+ *             iterations"): every entry goes to its nearest centre (ties to the
+ *             lower), each centre becomes its cluster's mean, an empty cluster keeps
+ *             its centre.  0 = the closed-form centres alone.
  *  codes_u,   required, uint32[m][ceil(n/16)]: 2-bit code of u_i (resp. vhat_i) at
  *  codes_v    bits 2*(i%16) of word i/16 of vector j's row; code c indexes the
  *             ascending centre table.
  *  centres_u, required, float[m][4] ascending: -(a1+a2), -|a1-a2|, |a1-a2|, a1+a2
- *  centres_v  with (a1, a2) = (c1, c2) for u and (d1, d2) for vhat.
+ *  centres_v  with (a1, a2) = (c1, c2) for u and (d1, d2) for vhat, or their
+ *             refinement when kmeans_iters > 0.
  *  coeffs     optional, float[m][4]: c1, c2, d1, d2 (block-0 step coefficients).
  *  u, vhat,   optional, float[m][n] (vector-major, contiguous): the factors u_k,
  *  resid      vhat_k and the residual r_k of Algorithm 1, x = u + P vhat + r.
- *  trace      optional, int8[m][4*iters][n]: sign(.) in {-1, 0, +1} that every
- *             atomic step applied to element i (natural order).  Test/debug
- *             output; enabling it does not change any other output bit.
+ *  trace      optional, int8[m][4*iters + 2*kmeans_iters][n]: rows 0..4k-1 hold the
+ *             sign(.) in {-1, 0, +1} every atomic step applied to element i (natural
+ *             order); rows 4k + 2t + f hold the cluster (0..3) of factor f (0 = u,
+ *             1 = vhat) in refinement iteration t.  Test/debug output; enabling it
+ *             does not change any other output bit.
  *  workspace  device scratch of ws_bytes >= kd_workspace_size(n).
  *
  * Vectors are processed two at a time (2j, 2j+1); each vector's results depend
  * only on its own data and its pair partner's (through rounding only). */
 kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
-                       int64_t ld, uint64_t sign_seed, int iters,
+                       int64_t ld, uint64_t sign_seed, int iters, int kmeans_iters,
                        uint32_t* codes_u, uint32_t* codes_v, float* centres_u, float* centres_v,
                        float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
                        void* workspace, size_t ws_bytes, void* stream);
@@ -123,7 +131,7 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
  *   - Non-finite inputs still set the device status word, which lives in the static
  *     array and is not readable through this ABI. */
 kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
-                              int64_t ld, uint64_t sign_seed, int iters,
+                              int64_t ld, uint64_t sign_seed, int iters, int kmeans_iters,
                               uint32_t* codes_u, uint32_t* codes_v, float* centres_u, float* centres_v,
                               float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
                               void* stream);

@@ -22,6 +22,9 @@ Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
                               step divisor ``N`` as printed.  Optional tie-follow.
 * ``centres`` / ``codes``  -- the closed-form centres +-c1 +-c2 (Sec. 2.1) and the
                               nearest-centre 2-bit code (Sec. 2.1, App. C).
+* ``kmeans_refine``        -- the "small number of k-means refinement iterations" that
+                              Sec. 2.1 runs from the closed-form centres: 1-D Lloyd steps
+                              with 4 centres, an empty cluster keeps its centre.
 * ``reconstruct``          -- dequantised ``W_hat = U_q + P V_q`` (App. C, Eq. 11).
 
 Parity pins (tests/test_oracle_pins.py) tie each function to something the paper
@@ -276,6 +279,40 @@ def dequantise(code: np.ndarray, cent: np.ndarray) -> np.ndarray:
     return np.asarray(cent, dtype=np.float64)[np.arange(M)[None, :], code]
 
 
+def kmeans_refine(values: np.ndarray, cent: np.ndarray, iters: int, follow: Optional[np.ndarray] = None,
+                  window: Optional[np.ndarray] = None):
+    """Lloyd refinement of each column's 4 centres (Sec. 2.1: the closed-form centres
+    initialise k-means, then a small number of refinement iterations run).
+
+    Per iteration: every entry goes to its nearest centre (ties to the lower index,
+    decided in float32 like :func:`codes`), then each centre becomes the float64
+    mean of its entries; a centre with no entries keeps its value.  Returns the
+    refined centres ``(M, 4)``, the final codes ``(N, M)`` and the number of followed
+    and hard-mismatched assignments.
+
+    ``follow`` (int, ``(iters, N, M)``) gives the device's assignment at each
+    iteration; where an entry lies within ``window[col]`` of a boundary the
+    device's code is used (both are nearest-centre within rounding)."""
+    v = np.asarray(values, dtype=np.float64)
+    c = np.array(cent, dtype=np.float64, copy=True)
+    N, M = v.shape
+    ties = hard = 0
+    for it in range(iters):
+        code = codes(v, c)
+        if follow is not None:
+            near = boundary_distance(v, c) <= window[None, :]
+            dev = follow[it].astype(np.int64)
+            ties += int((near & (dev != code)).sum())
+            hard += int((~near & (dev != code)).sum())
+            code = np.where(near, dev, code)
+        for q in range(4):
+            member = code == q
+            cnt = member.sum(axis=0)
+            tot = np.where(member, v, 0.0).sum(axis=0)
+            c[:, q] = np.where(cnt > 0, tot / np.maximum(cnt, 1), c[:, q])
+    return c, codes(v, c), ties, hard
+
+
 def reconstruct(code_u: np.ndarray, code_v: np.ndarray, cent_u: np.ndarray, cent_v: np.ndarray,
                 eps: np.ndarray) -> np.ndarray:
     """Dequantised weight ``W_hat = U_q + P V_q`` (App. C: dense re-materialisation)."""
@@ -295,14 +332,18 @@ class Quantised:
 
 
 def quantise(x: np.ndarray, seed: int, iters: int, follow: Optional[np.ndarray] = None,
-             tau_abs: Optional[np.ndarray] = None) -> Quantised:
+             tau_abs: Optional[np.ndarray] = None, kmeans_iters: int = 0) -> Quantised:
     """Decompose every column (Alg. 1), then code each factor with its closed-form
-    centres (Sec. 2.1): u with (c1, c2), vhat with (d1, d2), zero refinement
-    iterations (reading c-6)."""
+    centres (Sec. 2.1): u with (c1, c2), vhat with (d1, d2); ``kmeans_iters`` Lloyd
+    refinement iterations from those centres (0 = the closed form alone)."""
     x = np.asarray(x, dtype=np.float64)
     eps = sign_mask(seed, x.shape[0])
     dec = decompose(x, eps, iters, follow=follow, tau_abs=tau_abs)
     cu = centres(dec.coeffs[0], dec.coeffs[1])
     cv = centres(dec.coeffs[2], dec.coeffs[3])
+    if kmeans_iters > 0:
+        cu, code_u, _, _ = kmeans_refine(dec.u, cu, kmeans_iters)
+        cv, code_v, _, _ = kmeans_refine(dec.vhat, cv, kmeans_iters)
+        return Quantised(dec=dec, centres_u=cu, centres_v=cv, codes_u=code_u, codes_v=code_v)
     return Quantised(dec=dec, centres_u=cu, centres_v=cv, codes_u=codes(dec.u, cu),
                      codes_v=codes(dec.vhat, cv))

@@ -135,10 +135,12 @@ kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host) {
 }
 
 kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m, int64_t ld,
-                       uint64_t sign_seed, int iters, uint32_t* codes_u, uint32_t* codes_v,
+                       uint64_t sign_seed, int iters, int kmeans_iters, uint32_t* codes_u, uint32_t* codes_v,
                        float* centres_u, float* centres_v, float* coeffs, float* u, float* vhat,
                        float* resid, int8_t* trace, void* workspace, size_t ws_bytes, void* stream) {
-  if (n <= 0 || m < 0 || iters < 0 || !valid_dtype(dtype) || !valid_layout(layout)) return KD_ERR_INVALID_ARG;
+  if (n <= 0 || m < 0 || iters < 0 || kmeans_iters < 0 || kmeans_iters > 64 || !valid_dtype(dtype) ||
+      !valid_layout(layout))
+    return KD_ERR_INVALID_ARG;
   const PlanOps* ops = plan_ops(n);
   if (!ops) return KD_ERR_UNSUPPORTED_N;
   if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
@@ -158,6 +160,7 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
   p.m = m;
   p.ld = ld;
   p.iters = iters;
+  p.kmeans_iters = kmeans_iters;
   p.codes_u = codes_u;
   p.codes_v = codes_v;
   p.centres_u = centres_u;

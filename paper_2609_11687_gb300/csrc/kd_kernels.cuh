@@ -70,6 +70,55 @@ __device__ __forceinline__ float2 team_sum(float2 v, float2* red, int lt, int& p
   }
 }
 
+// Sum of K (a power of two <= 32) per-thread values over the team; every thread
+// receives all K totals in `tot` (fixed summation order: deterministic).
+// Whole-warp teams: butterfly reduce-scatter (K - 1 shuffles, then one shuffle per
+// remaining lane bit) leaves lane l with its warp's total of value l % K, then a
+// fixed-order sum over warps through `scratch` (K (NW + 1) floats of shared
+// memory).  Narrower teams: butterfly all-reduce over the team's lanes.
+template <class PL, int K>
+__device__ __forceinline__ void team_sum_k(float (&v)[K], float (&tot)[K], float* scratch, int lt) {
+  static_assert(K >= 1 && K <= 32 && (K & (K - 1)) == 0, "K must be a power of two <= 32");
+  if constexpr (PL::T < 32) {
+#pragma unroll
+    for (int off = PL::T / 2; off > 0; off >>= 1) {
+#pragma unroll
+      for (int i = 0; i < K; ++i) v[i] = __fadd_rn(v[i], __shfl_xor_sync(0xffffffffu, v[i], off));
+    }
+#pragma unroll
+    for (int i = 0; i < K; ++i) tot[i] = v[i];
+  } else {
+    const int lane = lt & 31;
+#pragma unroll
+    for (int k = K / 2; k >= 1; k >>= 1) {
+#pragma unroll
+      for (int i = 0; i < k; ++i) {
+        const bool hi = (lane & k) != 0;
+        const float send = hi ? v[i] : v[i + k];
+        const float keep = hi ? v[i + k] : v[i];
+        v[i] = __fadd_rn(keep, __shfl_xor_sync(0xffffffffu, send, k));
+      }
+    }
+#pragma unroll
+    for (int off = K; off < 32; off <<= 1) v[0] = __fadd_rn(v[0], __shfl_xor_sync(0xffffffffu, v[0], off));
+    // lane l now holds its warp's total of value l % K
+    float* wpart = scratch;             // [NW][K]
+    float* fin = scratch + K * PL::NW;  // [K]
+    if (lane < K) wpart[(lt >> 5) * K + lane] = v[0];
+    team_sync<PL>();
+    if (lt < K) {
+      float t = wpart[lt];
+#pragma unroll
+      for (int w = 1; w < PL::NW; ++w) t = __fadd_rn(t, wpart[w * K + lt]);
+      fin[lt] = t;
+    }
+    team_sync<PL>();
+#pragma unroll
+    for (int i = 0; i < K; ++i) tot[i] = fin[i];
+    team_sync<PL>();
+  }
+}
+
 // Shared memory of a CTA: [twiddle table (if staged)][team 0 buffer | red][team 1 ...].
 // Copies the table in and returns this team's buffer.
 template <class PL>
@@ -121,6 +170,7 @@ struct DecParams {
   int dtype, layout;
   int64_t n, m, ld;
   int iters;
+  int kmeans_iters;
   uint32_t* codes_u;
   uint32_t* codes_v;
   float* centres_u;
@@ -159,7 +209,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
   Xform<PL> xf;
   xf.init(buf, tw, p.eps, lt);
   int parity = 0;
-  const int nsteps = 4 * p.iters;
+  const int nsteps = 4 * p.iters + 2 * p.kmeans_iters;  // trace rows per vector
 
   float2 uu_reg[PL::UMODE == UREG ? E : 1];
   // u outside registers: per-team workspace slot (global) or shared memory after red
@@ -378,22 +428,100 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
       }
     }
 
-    // ---- 2-bit codes: nearest of the closed-form centres, ties low ----
-    const float muA = fmaxf(coef[0].x, coef[1].x), muB = fmaxf(coef[0].y, coef[1].y);
-    const float mvA = fmaxf(coef[2].x, coef[3].x), mvB = fmaxf(coef[2].y, coef[3].y);
+    // ---- centres: closed form +-a1 +-a2 (Sec. 2.1), then optional Lloyd refinement ----
+    // cen[f][c][q]: factor f (0 = u, 1 = vhat), vector c (0 = A, 1 = B), ascending centre q
+    float cen[2][2][4];
+    {
+      const float a1[2][2] = {{coef[0].x, coef[0].y}, {coef[2].x, coef[2].y}};
+      const float a2[2][2] = {{coef[1].x, coef[1].y}, {coef[3].x, coef[3].y}};
+#pragma unroll
+      for (int f = 0; f < 2; ++f)
+#pragma unroll
+        for (int c = 0; c < 2; ++c) {
+          const float outer = __fadd_rn(a1[f][c], a2[f][c]);
+          const float inner = fabsf(__fsub_rn(a1[f][c], a2[f][c]));
+          cen[f][c][0] = -outer;
+          cen[f][c][1] = -inner;
+          cen[f][c][2] = inner;
+          cen[f][c][3] = outer;
+        }
+    }
+    // decision boundaries: closed form uses -max(a1,a2), 0, +max(a1,a2) exactly
+    float bnd[2][2][3];
+#pragma unroll
+    for (int f = 0; f < 2; ++f)
+#pragma unroll
+      for (int c = 0; c < 2; ++c) {
+        const float mm = fmaxf(f ? (c ? coef[2].y : coef[2].x) : (c ? coef[0].y : coef[0].x),
+                               f ? (c ? coef[3].y : coef[3].x) : (c ? coef[1].y : coef[1].x));
+        bnd[f][c][0] = -mm;
+        bnd[f][c][1] = 0.f;
+        bnd[f][c][2] = mm;
+      }
+    auto code_of = [](float x, const float (&b)[3]) -> int { return (x > b[0]) + (x > b[1]) + (x > b[2]); };
+    auto val = [&](int j, int f, int c) -> float {
+      if (f == 0) {
+        const float2 uj = u_at(j);
+        return c ? uj.y : uj.x;
+      }
+      return c ? vh[j].y : vh[j].x;
+    };
+    {
+      for (int it = 0; it < p.kmeans_iters; ++it) {
+        // one factor at a time (keeps 16 accumulators live, not 32)
+#pragma unroll
+        for (int f = 0; f < 2; ++f) {
+          // per-thread sums [0, 8) and counts [8, 16) per (vector, centre)
+          float acc[16];
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+#pragma unroll
+          for (int j = 0; j < E; ++j) {
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+              const float x = val(j, f, c);
+              const int q = code_of(x, bnd[f][c]);
+              if constexpr (TRACE) {
+                if (tracing && (c == 0 || hasB)) {
+                  const int nat = nat_of<N>(lt + j * T);
+                  (c ? trB : trA)[(int64_t)(4 * p.iters + 2 * it + f) * N + nat] = (int8_t)q;
+                }
+              }
+#pragma unroll
+              for (int qq = 0; qq < 4; ++qq) {
+                const bool hit = (q == qq);
+                acc[c * 4 + qq] = __fadd_rn(acc[c * 4 + qq], hit ? x : 0.f);
+                acc[8 + c * 4 + qq] = __fadd_rn(acc[8 + c * 4 + qq], hit ? 1.f : 0.f);
+              }
+            }
+          }
+          float tot[16];
+          team_sum_k<PL, 16>(acc, tot, reinterpret_cast<float*>(red), lt);
+#pragma unroll
+          for (int c = 0; c < 2; ++c) {
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+              const float n_ = tot[8 + c * 4 + qq];
+              if (n_ > 0.f) cen[f][c][qq] = __fdiv_rn(tot[c * 4 + qq], n_);
+            }
+#pragma unroll
+            for (int qq = 0; qq < 3; ++qq)
+              bnd[f][c][qq] = __fmul_rn(0.5f, __fadd_rn(cen[f][c][qq], cen[f][c][qq + 1]));
+          }
+        }
+      }
+    }
+
+    // ---- 2-bit codes: nearest centre, ties low ----
     team_sync<PL>();  // everyone is done with buf
     uint8_t* cb = reinterpret_cast<uint8_t*>(buf);
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
-      auto code = [](float x, float mm) -> uint8_t {
-        return (uint8_t)((x > -mm) + (x > 0.f) + (x > mm));
-      };
-      const float2 uj = u_at(j);
-      cb[0 * N + nat] = code(uj.x, muA);
-      cb[1 * N + nat] = code(uj.y, muB);
-      cb[2 * N + nat] = code(vh[j].x, mvA);
-      cb[3 * N + nat] = code(vh[j].y, mvB);
+      cb[0 * N + nat] = (uint8_t)code_of(val(j, 0, 0), bnd[0][0]);
+      cb[1 * N + nat] = (uint8_t)code_of(val(j, 0, 1), bnd[0][1]);
+      cb[2 * N + nat] = (uint8_t)code_of(val(j, 1, 0), bnd[1][0]);
+      cb[3 * N + nat] = (uint8_t)code_of(val(j, 1, 1), bnd[1][1]);
     }
     team_sync<PL>();
     constexpr int WPV = N / 16;  // words per vector (N % 16 == 0 for every plan)
@@ -423,12 +551,13 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
           const float c1 = v2 ? coef[0].y : coef[0].x, c2 = v2 ? coef[1].y : coef[1].x;
           const float d1 = v2 ? coef[2].y : coef[2].x, d2 = v2 ? coef[3].y : coef[3].x;
           const float f = sc[v2];
-          const float uo = __fmul_rn(__fadd_rn(c1, c2), f), ui = __fmul_rn(fabsf(__fsub_rn(c1, c2)), f);
-          const float vo = __fmul_rn(__fadd_rn(d1, d2), f), vi = __fmul_rn(fabsf(__fsub_rn(d1, d2)), f);
           float* cu = p.centres_u + col * 4;
           float* cv = p.centres_v + col * 4;
-          cu[0] = -uo; cu[1] = -ui; cu[2] = ui; cu[3] = uo;
-          cv[0] = -vo; cv[1] = -vi; cv[2] = vi; cv[3] = vo;
+#pragma unroll
+          for (int qq = 0; qq < 4; ++qq) {
+            cu[qq] = __fmul_rn(cen[0][v2][qq], f);
+            cv[qq] = __fmul_rn(cen[1][v2][qq], f);
+          }
           if (p.coeffs) {
             float* co = p.coeffs + col * 4;
             co[0] = __fmul_rn(c1, f); co[1] = __fmul_rn(c2, f);

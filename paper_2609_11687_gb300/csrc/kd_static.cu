@@ -60,7 +60,8 @@ cudaError_t scratch_on_current_device(void** out) {
 }  // namespace kd
 
 extern "C" kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
-                                         int64_t ld, uint64_t sign_seed, int iters, uint32_t* codes_u,
+                                         int64_t ld, uint64_t sign_seed, int iters, int kmeans_iters,
+                                         uint32_t* codes_u,
                                          uint32_t* codes_v, float* centres_u, float* centres_v, float* coeffs,
                                          float* u, float* vhat, float* resid, int8_t* trace, void* stream) {
   if (n > kd::kStaticMaxN) return KD_ERR_WORKSPACE;
@@ -70,6 +71,7 @@ extern "C" kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layou
   if (need > kd::kStaticBytes) return KD_ERR_WORKSPACE;
   void* scratch = nullptr;
   if (kd::scratch_on_current_device(&scratch) != cudaSuccess) return KD_ERR_CUDA;
-  return kd_decompose(w, dtype, layout, n, m, ld, sign_seed, iters, codes_u, codes_v, centres_u, centres_v,
+  return kd_decompose(w, dtype, layout, n, m, ld, sign_seed, iters, kmeans_iters, codes_u, codes_v, centres_u,
+                      centres_v,
                       coeffs, u, vhat, resid, trace, scratch, kd::kStaticBytes, stream);
 }

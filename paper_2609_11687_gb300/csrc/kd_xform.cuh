@@ -83,7 +83,9 @@ struct Plan {
   static constexpr int THREADS = T * Q;
   static constexpr int NW = (T + 31) / 32;  // warps per team
   static constexpr int BUF = (N + N / 16 + N / 256 + 8 + 15) / 16 * 16;  // padded float2 slots per team
-  static constexpr int RED = 4 * (NW > 1 ? NW : 1);           // float2 reduction slots per team
+  // float2 reduction slots per team: ping-pong partials of team_sum, or the
+  // 16-value reduction of the k-means refinement (16 (NW + 1) floats = 8 (NW + 1) float2)
+  static constexpr int RED = (4 * NW > 8 * (NW + 1)) ? 4 * NW : 8 * (NW + 1);
   static constexpr int USL = (UMODE_ == 2) ? N : 0;            // float2 slots of u per team (shared)
   // M in registers: one last-pass group per thread, partner at lane ^ HALF
 #ifdef KD_NO_PAIRED

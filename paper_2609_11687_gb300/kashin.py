@@ -49,7 +49,7 @@ def _load() -> ctypes.CDLL:
     lib.kd_workspace_size.restype = c_sz
     lib.kd_signs.argtypes = [c_u64, c_i64, c_vp]
     lib.kd_signs.restype = c_int
-    lib.kd_decompose.argtypes = [c_vp, c_int, c_int, c_i64, c_i64, c_i64, c_u64, c_int,
+    lib.kd_decompose.argtypes = [c_vp, c_int, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_int,
                                  c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_sz, c_vp]
     lib.kd_decompose.restype = c_int
     lib.kd_apply_p.argtypes = [c_vp, c_vp, c_i64, c_i64, c_u64, c_vp, c_sz, c_vp]
@@ -99,11 +99,11 @@ def kd_signs(sign_seed: int, n: int) -> np.ndarray:
     return out
 
 
-def kd_decompose(w, dtype, layout, n, m, ld, sign_seed, iters, codes_u, codes_v, centres_u, centres_v,
-                 coeffs, u, vhat, resid, trace, workspace, ws_bytes, stream) -> int:
+def kd_decompose(w, dtype, layout, n, m, ld, sign_seed, iters, kmeans_iters, codes_u, codes_v, centres_u,
+                 centres_v, coeffs, u, vhat, resid, trace, workspace, ws_bytes, stream) -> int:
     return lib.kd_decompose(w, dtype, layout, n, m, ld, ctypes.c_uint64(int(sign_seed) & ((1 << 64) - 1)),
-                            iters, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat, resid, trace,
-                            workspace, ws_bytes, stream)
+                            iters, kmeans_iters, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat, resid,
+                            trace, workspace, ws_bytes, stream)
 
 
 def kd_apply_p(x, y, n, m, sign_seed, workspace, ws_bytes, stream) -> int:
@@ -177,13 +177,14 @@ class Decomposed:
     u: "object"           # float32 (m, n) or None
     vhat: "object"
     resid: "object"
-    trace: "object"       # int8 (m, 4*iters, n) or None
+    trace: "object"       # int8 (m, 4*iters + 2*kmeans_iters, n) or None
 
 
 def decompose(w, iters: int, sign_seed: int, layout: str = "rows", factors: bool = False,
               coeffs: bool = True, trace: bool = False, workspace: Optional[Workspace] = None,
-              out: Optional[Decomposed] = None, stream=None) -> Decomposed:
-    """Decompose every vector of ``w`` (Alg. 1) and 2-bit code both factors.
+              out: Optional[Decomposed] = None, stream=None, kmeans_iters: int = 0) -> Decomposed:
+    """Decompose every vector of ``w`` (Alg. 1) and 2-bit code both factors
+    (closed-form centres, then ``kmeans_iters`` Lloyd refinement iterations).
 
     ``layout='rows'``: ``w`` is (m, n), vector j = ``w[j]`` (nn.Linear weight).
     ``layout='columns'``: ``w`` is (n, m), vector j = ``w[:, j]`` (the paper's W).
@@ -211,9 +212,9 @@ def decompose(w, iters: int, sign_seed: int, layout: str = "rows", factors: bool
             u=torch.empty((m, n), **f32) if factors else None,
             vhat=torch.empty((m, n), **f32) if factors else None,
             resid=torch.empty((m, n), **f32) if factors else None,
-            trace=torch.empty((m, 4 * iters, n), dtype=torch.int8, device=dev) if trace else None)
+            trace=torch.empty((m, 4 * iters + 2 * kmeans_iters, n), dtype=torch.int8, device=dev) if trace else None)
     ws = workspace if workspace is not None else Workspace(n, dev)
-    st = kd_decompose(w.data_ptr(), _dtype_code(w.dtype), lay, n, m, ld, sign_seed, int(iters),
+    st = kd_decompose(w.data_ptr(), _dtype_code(w.dtype), lay, n, m, ld, sign_seed, int(iters), int(kmeans_iters),
                       _ptr(out.codes_u), _ptr(out.codes_v), _ptr(out.centres_u), _ptr(out.centres_v),
                       _ptr(out.coeffs), _ptr(out.u), _ptr(out.vhat), _ptr(out.resid), _ptr(out.trace),
                       ws.ptr, ws.nbytes, _stream(stream))

@@ -75,7 +75,7 @@ def _rel_inf(a, b):
     return float(out.max()) if out.size else 0.0
 
 
-def compare(x: np.ndarray, seed: int, iters: int, dev: dict, P_oracle=None) -> ParityReport:
+def compare(x: np.ndarray, seed: int, iters: int, dev: dict, P_oracle=None, kmeans_iters: int = 0) -> ParityReport:
     """x: (N, M) float64 inputs (exact values the device saw).  dev: numpy arrays
     from the device, vector-major: u, vhat, resid (M, N) float32, coeffs (M, 4),
     centres_u/centres_v (M, 4), codes_u/codes_v (M, N) int, trace (M, 4k, N) int8."""
@@ -83,13 +83,24 @@ def compare(x: np.ndarray, seed: int, iters: int, dev: dict, P_oracle=None) -> P
     eps = ko.sign_mask(seed, N)
     P = P_oracle if P_oracle is not None else ko.POperator(N, eps)
     xmax = np.abs(x).max(axis=0)
-    follow = np.transpose(dev["trace"], (1, 2, 0)).astype(np.int8)   # (4k, N, M)
+    trace = np.transpose(dev["trace"], (1, 2, 0)).astype(np.int8)    # (4k + 2 kmeans, N, M)
+    follow = trace[:4 * iters]
     floor = FLOOR * 2.0 ** -24 * np.linalg.norm(x, axis=0)
     d = ko.decompose(x, eps, iters, follow=follow, tau_abs=TAU * xmax, P=P, follow_floor=floor)
     cu = ko.centres(d.coeffs[0], d.coeffs[1])
     cv = ko.centres(d.coeffs[2], d.coeffs[3])
-    code_u = ko.codes(d.u, cu)
-    code_v = ko.codes(d.vhat, cv)
+    km_hard = 0
+    if kmeans_iters > 0:
+        # Lloyd refinement (Sec. 2.1) following the device's assignment near a boundary
+        km = trace[4 * iters:].reshape(kmeans_iters, 2, N, M)
+        wu = CODE_WINDOW * np.abs(cu[:, 3])
+        wv = CODE_WINDOW * np.abs(cv[:, 3])
+        cu, code_u, _, h1 = ko.kmeans_refine(d.u, cu, kmeans_iters, follow=km[:, 0], window=wu)
+        cv, code_v, _, h2 = ko.kmeans_refine(d.vhat, cv, kmeans_iters, follow=km[:, 1], window=wv)
+        km_hard = h1 + h2
+    else:
+        code_u = ko.codes(d.u, cu)
+        code_v = ko.codes(d.vhat, cv)
 
     u_g = dev["u"].T.astype(np.float64)
     v_g = dev["vhat"].T.astype(np.float64)
@@ -121,15 +132,16 @@ def compare(x: np.ndarray, seed: int, iters: int, dev: dict, P_oracle=None) -> P
     Pv = P(v_g)
     recon = np.linalg.norm(x - u_g - Pv - r_g, axis=0) / np.where(np.linalg.norm(x, axis=0) > 0,
                                                                   np.linalg.norm(x, axis=0), 1)
-    return ParityReport(n=N, m=M, hard=d.hard_mismatches, ties=d.ties, tie_flips=d.tie_flips, u_err=u_err,
+    return ParityReport(n=N, m=M, hard=d.hard_mismatches + km_hard, ties=d.ties, tie_flips=d.tie_flips, u_err=u_err,
                         v_err=v_err, coef_err=coef_err, cent_err=cent_err, code_diff=diff,
                         code_diff_outside=outside, code_near=near_total, recon_err=float(recon.max()),
                         entries=2 * N * M)
 
 
-def device_outputs(kd, w_dev, iters, seed, trace=True, layout="rows"):
+def device_outputs(kd, w_dev, iters, seed, trace=True, layout="rows", kmeans_iters=0):
     """Run kd_decompose with every optional output and return numpy arrays."""
-    out = kd.decompose(w_dev, iters, seed, layout=layout, factors=True, coeffs=True, trace=trace)
+    out = kd.decompose(w_dev, iters, seed, layout=layout, factors=True, coeffs=True, trace=trace,
+                       kmeans_iters=kmeans_iters)
     n = out.u.shape[1]
     import torch
     torch.cuda.synchronize()

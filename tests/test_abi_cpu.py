@@ -73,24 +73,27 @@ def test_workspace_size_register_plans(kd):
 def test_argument_validation_without_gpu(kd):
     null = None
     # unsupported length
-    st = kd.kd_decompose(1, 0, 0, 100, 4, 100, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20, null)
+    st = kd.kd_decompose(1, 0, 0, 100, 4, 100, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20, null)
     assert st == kd.KD_ERR_UNSUPPORTED_N
+    # out-of-range refinement count
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 65, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
     # negative iterations / bad dtype / bad layout / ld too small
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, -1, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, -1, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
                            null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_decompose(1, 7, 0, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+    assert kd.kd_decompose(1, 7, 0, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
                            null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_decompose(1, 0, 5, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+    assert kd.kd_decompose(1, 0, 5, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
                            null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 255, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 255, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
                            null) == kd.KD_ERR_INVALID_ARG
     # missing required outputs
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, null, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, null, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
                            null) == kd.KD_ERR_INVALID_ARG
     # workspace missing / too small
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, null, 1 << 20,
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, null, 1 << 20,
                            null) == kd.KD_ERR_WORKSPACE
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 1, 1, 1, 1, null, null, null, null, null, 1, 16,
+    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 16,
                            null) == kd.KD_ERR_WORKSPACE
     assert kd.kd_apply_p(1, 1, 256, 2, 0, null, 0, null) == kd.KD_ERR_WORKSPACE
     assert kd.kd_apply_p(null, 1, 256, 2, 0, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG

@@ -69,14 +69,14 @@ def test_apply_p_is_involution(kd, torch_mod, n):
 # Full decomposition parity
 # ---------------------------------------------------------------------------
 
-def _parity(kd, torch, G_cpu, seed, iters=ITERS, layout="rows"):
+def _parity(kd, torch, G_cpu, seed, iters=ITERS, layout="rows", kmeans_iters=0):
     """G_cpu: (M, N) tensor (vector-major) on the CPU holding the exact inputs."""
     w = G_cpu.cuda()
     if layout == "columns":
         w = G_cpu.t().contiguous().cuda()
-    dev = parity.device_outputs(kd, w, iters, seed, trace=True, layout=layout)
+    dev = parity.device_outputs(kd, w, iters, seed, trace=True, layout=layout, kmeans_iters=kmeans_iters)
     x = G_cpu.to(torch.float64).numpy().T  # (N, M)
-    rep = parity.compare(x, seed, iters, dev)
+    rep = parity.compare(x, seed, iters, dev, kmeans_iters=kmeans_iters)
     return rep, dev
 
 
@@ -193,6 +193,39 @@ def test_deterministic(kd, torch_mod):
     b = kd.decompose(w, ITERS, 1)
     torch.cuda.synchronize()
     assert torch.equal(a.codes_u, b.codes_u) and torch.equal(a.centres_v, b.centres_v)
+
+
+# ---------------------------------------------------------------------------
+# k-means refinement of the centres (Sec. 2.1)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("n,m,kiters", [(256, 16, 3), (768, 9, 1), (3072, 6, 3), (4096, 10, 5), (11008, 4, 3)])
+def test_kmeans_refinement_parity(kd, torch_mod, n, m, kiters):
+    torch = torch_mod
+    G = _rand(torch, (m, n), seed=n + 3, dtype=torch.float16)
+    rep, dev = _parity(kd, torch, G.float(), seed=n, kmeans_iters=kiters)
+    print(rep)
+    rep.check()
+    # refinement lowers each factor's within-cluster squared error vs the closed form
+    closed = kd.decompose(G.cuda(), ITERS, n, factors=True)
+    torch.cuda.synchronize()
+    def sse(vals, cent, words):
+        code = kd.unpack_codes(words, n)
+        c = cent.cpu().numpy().astype(np.float64)
+        return ((vals.cpu().numpy().astype(np.float64) - c[np.arange(m)[:, None], code]) ** 2).sum(1)
+    assert np.all(sse(closed.u, torch.from_numpy(dev["centres_u"]), torch.from_numpy(dev["words_u"]))
+                  <= sse(closed.u, closed.centres_u, closed.codes_u) * (1 + 1e-5))
+
+
+def test_kmeans_zero_iters_is_closed_form(kd, torch_mod):
+    torch = torch_mod
+    w = _rand(torch, (6, 4096), seed=2, dtype=torch.float16).cuda()
+    a = kd.decompose(w, ITERS, 5)
+    b = kd.decompose(w, ITERS, 5, kmeans_iters=0)
+    c = kd.decompose(w, ITERS, 5, kmeans_iters=2)
+    torch.cuda.synchronize()
+    assert torch.equal(a.centres_u, b.centres_u) and torch.equal(a.codes_v, b.codes_v)
+    assert not torch.equal(a.centres_u, c.centres_u)
 
 
 # ---------------------------------------------------------------------------

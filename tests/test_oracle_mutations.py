@@ -26,6 +26,10 @@ MUTANTS = {
     "codes_tie_upper": ("out += (v32 > b[None, :, i])", "out += (v32 >= b[None, :, i])"),
     "pack_shift": ("<< np.uint64(2 * (i % 16))", "<< np.uint64(2 * (15 - i % 16))"),
     "mask_low_bit": ("out[j] = -1.0 if (z >> 63) else 1.0", "out[j] = -1.0 if (z & 1) else 1.0"),
+    "kmeans_empty_to_zero": ("c[:, q] = np.where(cnt > 0, tot / np.maximum(cnt, 1), c[:, q])",
+                             "c[:, q] = tot / np.maximum(cnt, 1)"),
+    "kmeans_sum_not_mean": ("c[:, q] = np.where(cnt > 0, tot / np.maximum(cnt, 1), c[:, q])",
+                            "c[:, q] = np.where(cnt > 0, tot, c[:, q])"),
     "reverse_schedule_u_second": ("for j in (1, 2):                     # two greedy steps from Q_N",
                                   "for j in ():"),
 }

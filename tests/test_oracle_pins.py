@@ -328,3 +328,50 @@ def test_follow_floor_gates_following():
     np.testing.assert_array_equal(gated.u, ref.u)
     open_gate = ko.decompose(x, eps, k, follow=planted, tau_abs=np.full(2, 1e9), follow_floor=np.zeros(2))
     assert open_gate.ties == 4 * k * N * 2
+
+
+# ---------------------------------------------------------------------------
+# k-means refinement (Sec. 2.1)
+# ---------------------------------------------------------------------------
+
+
+def test_kmeans_hand_worked():
+    """values -5,-4 | -1 | 0.5, 1.5 | 6 with centres (-4, -1, 1, 4): one Lloyd step
+    gives means -4.5, -1, 1, 6 (assignment by the midpoints -2.5, 0, 2.5)."""
+    vals = np.array([-5.0, -4.0, -1.0, 0.5, 1.5, 6.0])[:, None]
+    cent = np.array([[-4.0, -1.0, 1.0, 4.0]])
+    c1, code, _, _ = ko.kmeans_refine(vals, cent, 1)
+    np.testing.assert_array_equal(c1[0], [-4.5, -1.0, 1.0, 6.0])
+    np.testing.assert_array_equal(code[:, 0], [0, 0, 1, 2, 2, 3])
+
+
+def test_kmeans_empty_cluster_keeps_centre_and_order():
+    vals = np.array([0.1, 0.2, 0.3])[:, None]
+    cent = np.array([[-3.0, -1.0, 1.0, 3.0]])
+    c1, _, _, _ = ko.kmeans_refine(vals, cent, 2)
+    np.testing.assert_allclose(c1[0], [-3.0, -1.0, 0.2, 3.0])
+    assert np.all(np.diff(c1[0]) > 0)
+
+
+def _sse(vals, cent):
+    code = ko.codes(vals, cent)
+    return ((vals - ko.dequantise(code, cent)) ** 2).sum(axis=0)
+
+
+def test_kmeans_sse_non_increasing_and_zero_iters():
+    """Lloyd steps never increase the within-cluster squared error; zero iterations
+    leave the closed-form centres (Sec. 2.1) untouched."""
+    N = 256
+    x = _gauss(N, 6, seed=12)
+    q0 = ko.quantise(x, 3, 4)
+    prev = _sse(q0.dec.u, q0.centres_u)
+    for k in (1, 2, 3, 6):
+        c, _, _, _ = ko.kmeans_refine(q0.dec.u, q0.centres_u, k)
+        cur = _sse(q0.dec.u, c)
+        assert np.all(cur <= prev * (1 + 1e-12))
+        prev = cur
+    c0, code0, _, _ = ko.kmeans_refine(q0.dec.u, q0.centres_u, 0)
+    np.testing.assert_array_equal(c0, q0.centres_u)
+    np.testing.assert_array_equal(code0, q0.codes_u)
+    q3 = ko.quantise(x, 3, 4, kmeans_iters=3)
+    assert np.all(_sse(q3.dec.u, q3.centres_u) <= _sse(q0.dec.u, q0.centres_u))

@@ -24,7 +24,7 @@ def env():
     lib = ctypes.CDLL(kd.LIB_PATH)
     vp, i64 = ctypes.c_void_p, ctypes.c_int64
     lib.kd_decompose_static.argtypes = [vp, ctypes.c_int, ctypes.c_int, i64, i64, i64, ctypes.c_uint64,
-                                        ctypes.c_int] + [vp] * 10
+                                        ctypes.c_int, ctypes.c_int] + [vp] * 10
     lib.kd_decompose_static.restype = ctypes.c_int
     return torch, kd, lib
 
@@ -38,7 +38,7 @@ def _static(torch, kd, lib, w, iters, seed):
     for k in ("u", "vhat", "resid"):
         o[k] = torch.empty((m, n), dtype=torch.float32, device="cuda")
     st = lib.kd_decompose_static(w.data_ptr(), kd._dtype_code(w.dtype), kd.KD_VEC_ROWS, n, m, w.stride(0),
-                                 seed, iters, o["codes_u"].data_ptr(), o["codes_v"].data_ptr(),
+                                 seed, iters, 0, o["codes_u"].data_ptr(), o["codes_v"].data_ptr(),
                                  o["centres_u"].data_ptr(), o["centres_v"].data_ptr(), o["coeffs"].data_ptr(),
                                  o["u"].data_ptr(), o["vhat"].data_ptr(), o["resid"].data_ptr(), None,
                                  torch.cuda.current_stream().cuda_stream)
@@ -68,7 +68,7 @@ def test_static_scratch_refuses_long_vectors(env):
     torch, kd, lib = env
     w = torch.zeros((2, 11008), dtype=torch.float16, device="cuda")
     dummy = torch.empty(64, dtype=torch.int32, device="cuda")
-    st = lib.kd_decompose_static(w.data_ptr(), kd.KD_F16, kd.KD_VEC_ROWS, 11008, 2, 11008, 0, 4,
+    st = lib.kd_decompose_static(w.data_ptr(), kd.KD_F16, kd.KD_VEC_ROWS, 11008, 2, 11008, 0, 4, 0,
                                  dummy.data_ptr(), dummy.data_ptr(), dummy.data_ptr(), dummy.data_ptr(),
                                  None, None, None, None, None, None)
     assert st == kd.KD_ERR_WORKSPACE
