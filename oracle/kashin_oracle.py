@@ -10,7 +10,7 @@ Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
 
 * ``dct2_matrix``          -- orthonormal DCT-II (Sec. 3.1, footnote on ``norm='ortho'``;
                               App. C footnote).  Row 0 carries the extra ``1/sqrt 2``
-                              that makes the matrix orthogonal (reading c-1).
+                              that makes the matrix orthogonal (the printed formula omits it).
 * ``sign_mask``            -- the per-matrix sign set ``epsilon`` (Sec. 3.1 ``T_E``;
                               App. C "generated once from a fixed seed").  The paper
                               does not name its generator; this build reads it as
@@ -26,6 +26,10 @@ Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
                               Sec. 2.1 runs from the closed-form centres: 1-D Lloyd steps
                               with 4 centres, an empty cluster keeps its centre.
 * ``reconstruct``          -- dequantised ``W_hat = U_q + P V_q`` (App. C, Eq. 11).
+* ``greedy_original``      -- Algorithm 2 (App. B), the original vector greedy algorithm
+                              that Fig. 2 compares against: one projection step per
+                              update on whichever of ``x`` and ``Q x`` has the larger
+                              ``l_1`` norm.
 
 Parity pins (tests/test_oracle_pins.py) tie each function to something the paper
 or mathematics fixes; the ``l_inf`` bound constant of Theorem 2 contains the
@@ -125,7 +129,7 @@ class Decomposition:
 
 
 def _sign(a: np.ndarray) -> np.ndarray:
-    """``sign`` with ``sign(0) = 0`` (reading c-2)."""
+    """``sign`` with ``sign(0) = 0``: an exact zero entry takes no step (the paper does not say)."""
     return np.sign(a)
 
 
@@ -208,6 +212,67 @@ def decompose(x: np.ndarray, eps: np.ndarray, iters: int, follow: Optional[np.nd
     norms[step] = np.linalg.norm(r, axis=0)
     return Decomposition(u=u, vhat=vhat, r=r, coeffs=coeffs, lambdas=lambdas, step_norms=norms,
                          ties=stats["ties"], tie_flips=stats["flips"], hard_mismatches=stats["hard"])
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 2: the original vector greedy algorithm (App. B)
+# ---------------------------------------------------------------------------
+
+
+@dataclasses.dataclass
+class GreedyOriginal:
+    u: np.ndarray           # (N,)
+    vhat: np.ndarray        # (N,), transform-domain factor; v = Q^T vhat
+    r: np.ndarray           # (N,) residual
+    norms: np.ndarray       # (updates + 1,): ||r||_2 before the first update, then after each
+    branch: np.ndarray      # (updates,): 0 = u-update, 1 = vhat-update
+    coeffs: np.ndarray      # (updates,): projection coefficient of every update
+
+
+def greedy_original(x: np.ndarray, Q, tol: float = 0.0, max_updates: int = 64) -> GreedyOriginal:
+    """Algorithm 2 on one vector ``x`` (float64) with the orthogonal operator ``Q``
+    (a callable; Fig. 2 compares with the same sign-randomised DCT ``P``, so
+    ``Q^T = Q``).  While ``||r|| >= tol`` and fewer than ``max_updates`` updates:
+
+    * if ``||r||_1 > ||Q r||_1``: ``s = sign(r)``, ``pi = (r . s / ||s||^2) s``,
+      ``u += pi``, ``r -= pi``;
+    * else: ``s = sign(Q r)``, ``pi = ((Q r) . s / ||s||^2) s``, ``vhat += pi``,
+      ``r -= Q^T pi``.
+
+    The printed listing writes the second projection as ``pi_x(Sign(Q x))``, i.e. with
+    ``x`` itself on the left of the inner product; it is taken here as the projection
+    of ``Q x`` (the only choice that makes the step the least-squares move along
+    ``Q^T s``, as the first branch is along ``s``).  ``||s||^2`` counts the non-zero
+    entries, so an exact zero is left alone as in Alg. 1.
+    """
+    r = np.asarray(x, dtype=np.float64).copy()
+    u = np.zeros_like(r)
+    vhat = np.zeros_like(r)
+    norms = [np.linalg.norm(r)]
+    branch = []
+    coeffs = []
+    while norms[-1] >= tol and len(branch) < max_updates:
+        y = Q(r)
+        if np.abs(r).sum() > np.abs(y).sum():
+            s = _sign(r)
+            nnz = float(s @ s)
+            c = float(r @ s) / nnz if nnz else 0.0
+            u = u + c * s
+            r = r - c * s
+            branch.append(0)
+        else:
+            s = _sign(y)
+            nnz = float(s @ s)
+            c = float(y @ s) / nnz if nnz else 0.0
+            vhat = vhat + c * s
+            r = r - Q(c * s)
+            branch.append(1)
+        coeffs.append(c)
+        norms.append(np.linalg.norm(r))
+        if c == 0.0:
+            break
+    return GreedyOriginal(u=u, vhat=vhat, r=r, norms=np.array(norms), branch=np.array(branch, dtype=np.int8),
+                          coeffs=np.array(coeffs))
 
 
 # ---------------------------------------------------------------------------

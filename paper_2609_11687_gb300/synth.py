@@ -161,6 +161,11 @@ def config5(layers: Sequence[int] = range(32)) -> List[MatrixSpec]:
     return out
 
 
+def gaussian_vectors(n: int, m: int = 1, seed: int = 0) -> MatrixSpec:
+    """Fig. 2's input: ``m`` vectors of length ``n`` drawn from N(0, I_n), fp32."""
+    return MatrixSpec(f"gauss{n}x{m}", n, m, seed=seed, dist="normal", std=1.0, dtype=torch.float32)
+
+
 CONFIGS = {1: config1, 2: config2, 3: config3, 4: config4, 5: config5}
 
 

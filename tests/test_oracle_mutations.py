@@ -30,6 +30,9 @@ MUTANTS = {
                              "c[:, q] = tot / np.maximum(cnt, 1)"),
     "kmeans_sum_not_mean": ("c[:, q] = np.where(cnt > 0, tot / np.maximum(cnt, 1), c[:, q])",
                             "c[:, q] = np.where(cnt > 0, tot, c[:, q])"),
+    "alg2_literal_projection": ("c = float(y @ s) / nnz if nnz else 0.0", "c = float(r @ s) / nnz if nnz else 0.0"),
+    "alg2_branch_reversed": ("if np.abs(r).sum() > np.abs(y).sum():", "if np.abs(r).sum() < np.abs(y).sum():"),
+    "alg2_v_update_without_Q": ("r = r - Q(c * s)", "r = r - c * s"),
     "reverse_schedule_u_second": ("for j in (1, 2):                     # two greedy steps from Q_N",
                                   "for j in ():"),
 }

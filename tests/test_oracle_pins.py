@@ -226,7 +226,7 @@ def test_zero_column_stays_zero():
 
 
 def test_zero_inputs_keep_sign_zero():
-    """sign(0) = 0 (reading c-2): an exact zero entry is left untouched by the
+    """sign(0) = 0 (the paper leaves it open): an exact zero entry is left untouched by the
     two Q_N steps of the first block."""
     x = _gauss(64, 1, seed=9)
     x[[3, 17, 40]] = 0.0
@@ -375,3 +375,46 @@ def test_kmeans_sse_non_increasing_and_zero_iters():
     np.testing.assert_array_equal(code0, q0.codes_u)
     q3 = ko.quantise(x, 3, 4, kmeans_iters=3)
     assert np.all(_sse(q3.dec.u, q3.centres_u) <= _sse(q0.dec.u, q0.centres_u))
+
+
+# ---------------------------------------------------------------------------
+# Algorithm 2 (App. B): the original vector greedy algorithm
+# ---------------------------------------------------------------------------
+
+def test_alg2_hand_worked_n2_swap():
+    """N = 2 with the exact swap P (eps = (+1, -1)) and x = (3, 1): ||x||_1 = ||P x||_1,
+    so both updates take the vhat branch.  First: P x = (1, 3), s = (1, 1),
+    coefficient 4/2 = 2, vhat = (2, 2), r = x - P (2, 2) = (1, -1).  Second:
+    P r = (-1, 1), s = (-1, 1), coefficient 2/2 = 1, vhat = (1, 3), r = 0."""
+    swap = lambda z: np.asarray(z, dtype=np.float64)[::-1].copy()
+    g = ko.greedy_original(np.array([3.0, 1.0]), swap, tol=1e-300, max_updates=8)
+    np.testing.assert_array_equal(g.branch, [1, 1])
+    np.testing.assert_array_equal(g.coeffs, [2.0, 1.0])
+    np.testing.assert_array_equal(g.vhat, [1.0, 3.0])
+    np.testing.assert_array_equal(g.u, [0.0, 0.0])
+    np.testing.assert_array_equal(g.r, [0.0, 0.0])
+    np.testing.assert_array_equal(g.norms, [np.sqrt(10.0), np.sqrt(2.0), 0.0])
+
+
+@pytest.mark.parametrize("seed", [0, 1, 2])
+def test_alg2_prefix_replay_branch_and_drop(seed):
+    """Replaying Algorithm 2 for t updates gives the residual r_t entering update t.
+    Update t must take the branch with the larger l1 norm of r_t and P r_t, and, with
+    no zero entries, lower ||r||^2 by exactly max(||r_t||_1, ||P r_t||_1)^2 / N (the
+    squared length of the projection onto the chosen sign vector); the factors must
+    reconstruct x exactly."""
+    N = 64
+    x = _gauss(N, 1, seed=40 + seed)[:, 0]
+    eps = ko.sign_mask(seed, N)
+    P = ko.POperator(N, eps)
+    T = 12
+    full = ko.greedy_original(x, P, tol=0.0, max_updates=T)
+    assert len(full.branch) == T
+    for t in range(T):
+        r_t = ko.greedy_original(x, P, tol=0.0, max_updates=t).r
+        l1_u, l1_v = np.abs(r_t).sum(), np.abs(P(r_t)).sum()
+        assert full.branch[t] == (0 if l1_u > l1_v else 1)
+        drop = full.norms[t] ** 2 - full.norms[t + 1] ** 2
+        np.testing.assert_allclose(drop, max(l1_u, l1_v) ** 2 / N, rtol=1e-9)
+    np.testing.assert_allclose(full.u + P(full.vhat) + full.r, x, atol=1e-12)
+    assert np.all(np.diff(full.norms) < 0)
