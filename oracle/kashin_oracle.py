@@ -26,6 +26,12 @@ Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
                               Sec. 2.1 runs from the closed-form centres: 1-D Lloyd steps
                               with 4 centres, an empty cluster keeps its centre.
 * ``reconstruct``          -- dequantised ``W_hat = U_q + P V_q`` (App. C, Eq. 11).
+* ``randomized_hadamard``  -- the randomized-Hadamard incoherence rotation that the
+                              Kashin-DCT+H pipeline applies to a weight matrix before the
+                              decomposition (Sec. 4): ``y = (I (x) H_b / sqrt b) diag(s) x``
+                              per vector, Sylvester ``H_b`` on blocks of ``b`` = the largest
+                              power of two dividing the length (at most 16384), signs ``s``
+                              from the same SplitMix64 sequence as ``epsilon``.
 * ``greedy_original``      -- Algorithm 2 (App. B), the original vector greedy algorithm
                               that Fig. 2 compares against: one projection step per
                               update on whichever of ``x`` and ``Q x`` has the larger
@@ -212,6 +218,55 @@ def decompose(x: np.ndarray, eps: np.ndarray, iters: int, follow: Optional[np.nd
     norms[step] = np.linalg.norm(r, axis=0)
     return Decomposition(u=u, vhat=vhat, r=r, coeffs=coeffs, lambdas=lambdas, step_norms=norms,
                          ties=stats["ties"], tie_flips=stats["flips"], hard_mismatches=stats["hard"])
+
+
+# ---------------------------------------------------------------------------
+# Randomized-Hadamard incoherence rotation (Sec. 4, Kashin-DCT+H)
+# ---------------------------------------------------------------------------
+
+RHT_MAX_BLOCK = 16384
+
+
+def hadamard_matrix(b: int) -> np.ndarray:
+    """Sylvester Hadamard matrix of order ``b`` (a power of two):
+    ``H_1 = [1]``, ``H_2k = [[H_k, H_k], [H_k, -H_k]]``."""
+    assert b >= 1 and (b & (b - 1)) == 0
+    H = np.ones((1, 1))
+    while H.shape[0] < b:
+        H = np.block([[H, H], [H, -H]])
+    return H
+
+
+def rht_block(n: int) -> int:
+    """Block length of the rotation for vectors of length ``n``: the largest power
+    of two dividing ``n``, capped at ``RHT_MAX_BLOCK``."""
+    b = n & -n
+    return min(b, RHT_MAX_BLOCK)
+
+
+def randomized_hadamard(x: np.ndarray, seed: int, inverse: bool = False) -> np.ndarray:
+    """Rotate every column of ``x`` (shape ``(n, m)`` or ``(n,)``), float64.
+
+    Forward: ``y = R x`` with ``R = (I_{n/b} (x) H_b / sqrt(b)) diag(s)``: flip signs
+    by ``s = sign_mask(seed, n)``, then an orthonormal Hadamard transform on each
+    contiguous block of ``b = rht_block(n)`` entries.  Inverse: ``R^T``, i.e. the
+    block transform first, then the sign flip (``H_b`` is symmetric).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    one = x.ndim == 1
+    if one:
+        x = x[:, None]
+    n = x.shape[0]
+    b = rht_block(n)
+    Hn = hadamard_matrix(b) / np.sqrt(b)
+    s = sign_mask(seed, n)[:, None]
+    z = x if inverse else s * x
+    y = np.empty_like(z)
+    for k in range(n // b):
+        y[k * b:(k + 1) * b] = Hn @ z[k * b:(k + 1) * b]
+    if inverse:
+        y = s * y
+    return y[:, 0] if one else y
 
 
 # ---------------------------------------------------------------------------

@@ -33,6 +33,17 @@ MUTANTS = {
     "alg2_literal_projection": ("c = float(y @ s) / nnz if nnz else 0.0", "c = float(r @ s) / nnz if nnz else 0.0"),
     "alg2_branch_reversed": ("if np.abs(r).sum() > np.abs(y).sum():", "if np.abs(r).sum() < np.abs(y).sum():"),
     "alg2_v_update_without_Q": ("r = r - Q(c * s)", "r = r - c * s"),
+    "rht_no_normalisation": ("Hn = hadamard_matrix(b) / np.sqrt(b)", "Hn = hadamard_matrix(b)"),
+    "rht_signs_after_transform": ("z = x if inverse else s * x\n    y = np.empty_like(z)\n"
+                                  "    for k in range(n // b):\n"
+                                  "        y[k * b:(k + 1) * b] = Hn @ z[k * b:(k + 1) * b]\n"
+                                  "    if inverse:\n        y = s * y",
+                                  "z = x\n    y = np.empty_like(z)\n"
+                                  "    for k in range(n // b):\n"
+                                  "        y[k * b:(k + 1) * b] = Hn @ z[k * b:(k + 1) * b]\n"
+                                  "    if True:\n        y = s * y"),
+    "rht_whole_vector_block": ("    b = n & -n\n    return min(b, RHT_MAX_BLOCK)", "    return n"),
+    "hadamard_wrong_sign_block": ("H = np.block([[H, H], [H, -H]])", "H = np.block([[H, H], [-H, H]])"),
     "reverse_schedule_u_second": ("for j in (1, 2):                     # two greedy steps from Q_N",
                                   "for j in ():"),
 }

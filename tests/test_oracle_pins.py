@@ -418,3 +418,61 @@ def test_alg2_prefix_replay_branch_and_drop(seed):
         np.testing.assert_allclose(drop, max(l1_u, l1_v) ** 2 / N, rtol=1e-9)
     np.testing.assert_allclose(full.u + P(full.vhat) + full.r, x, atol=1e-12)
     assert np.all(np.diff(full.norms) < 0)
+
+
+# ---------------------------------------------------------------------------
+# Randomized-Hadamard rotation (Sec. 4, Kashin-DCT+H)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("b", [1, 2, 4, 16, 256, 1024])
+def test_hadamard_matches_scipy_sylvester(b):
+    scipy_linalg = pytest.importorskip("scipy.linalg")
+    np.testing.assert_array_equal(ko.hadamard_matrix(b), scipy_linalg.hadamard(b))
+
+
+def test_hadamard_orthogonal_brute_force():
+    for b in (2, 8, 64):
+        H = ko.hadamard_matrix(b)
+        np.testing.assert_array_equal(H @ H.T, b * np.eye(b))
+
+
+def test_rht_block_lengths():
+    assert [ko.rht_block(n) for n in (16, 256, 768, 3072, 4096, 11008, 14336, 16384, 32768, 40)] == \
+        [16, 256, 256, 1024, 4096, 256, 2048, 16384, 16384, 8]
+
+
+def test_rht_n2_hand_worked():
+    """n = 2, b = 2: y = [[1, 1], [1, -1]] / sqrt 2 applied to (s0 x0, s1 x1), signs
+    first (the sign set comes from the SplitMix64 sequence pinned above).  For
+    x = (3, 1): y = (3 s0 + s1, 3 s0 - s1) / sqrt 2; the inverse maps it back."""
+    for seed in range(8):
+        s0, s1 = ko.sign_mask(seed, 2)
+        y = ko.randomized_hadamard(np.array([3.0, 1.0]), seed)
+        np.testing.assert_allclose(y, np.array([3 * s0 + s1, 3 * s0 - s1]) / np.sqrt(2.0), rtol=0, atol=1e-15)
+        np.testing.assert_allclose(ko.randomized_hadamard(y, seed, inverse=True), [3.0, 1.0], rtol=0, atol=1e-15)
+    # both sign orders occur among these seeds, so the order of flip and transform is exercised
+    assert len({tuple(ko.sign_mask(sd, 2)) for sd in range(8)}) >= 3
+
+
+def test_rht_spike_is_flat_and_blocks_independent():
+    """A unit spike at j spreads to +-1/sqrt(b) over j's block and nowhere else
+    (incoherence); the transform acts block by block (n = 768 = 3 blocks of 256)."""
+    n, seed = 768, 11
+    for j in (0, 300, 767):
+        e = np.zeros(n)
+        e[j] = 1.0
+        y = ko.randomized_hadamard(e, seed)
+        blk = j // 256
+        inside = y[blk * 256:(blk + 1) * 256]
+        np.testing.assert_allclose(np.abs(inside), 1.0 / 16.0, rtol=0, atol=1e-15)
+        assert np.count_nonzero(np.delete(y, np.s_[blk * 256:(blk + 1) * 256])) == 0
+
+
+def test_rht_orthogonal_roundtrip():
+    x = _gauss(4096, 3, seed=8)
+    y = ko.randomized_hadamard(x, 5)
+    np.testing.assert_allclose(np.linalg.norm(y, axis=0), np.linalg.norm(x, axis=0), rtol=1e-13)
+    np.testing.assert_allclose(ko.randomized_hadamard(y, 5, inverse=True), x, rtol=0, atol=1e-13)
+    # the inverse is the transpose: <R x, z> = <x, R^T z>
+    z = _gauss(4096, 3, seed=9)
+    np.testing.assert_allclose((y * z).sum(0), (x * ko.randomized_hadamard(z, 5, inverse=True)).sum(0), rtol=1e-12)
