@@ -282,6 +282,9 @@ def run_gpu(args) -> dict:
     if args.kmeans_iters == 0:
         refinement = measure_refinement(kd, torch, layers[my_layers[-1]], outs, wss, iters, stream, dur)
 
+    # randomized-Hadamard pre-rotation (Kashin-DCT+H), HBM roofline
+    rotation = measure_rht(kd, torch, layers[my_layers[-1]], stream)
+
     # end to end: pinned host input, H2D + decompose + D2H codes/centres each step
     e2e = None
     if not args.skip_e2e:
@@ -299,11 +302,12 @@ def run_gpu(args) -> dict:
                    "l2": "inputs larger than L2 (405 MB per step, distinct layer every step)",
                    "parallelism": f"dp{world} (layers sharded over ranks, no exchange)"},
         "roofline": roofline,
-        "gpu_launches": args.steps * 7 * 2,
+        "gpu_launches": args.steps * 7 * 2,   # decompose + table set-up per matrix
         "clocks": clk,
     }
     if refinement is not None:
         result["kmeans_refinement"] = refinement
+    result["hadamard_rotation"] = rotation
     if e2e is not None:
         result["e2e"] = e2e
     if rank == 0 and world == 1 and not args.skip_cpu:
@@ -315,6 +319,46 @@ def run_gpu(args) -> dict:
 
 
 KM_PROBE = 3
+RHT_SEED = 0x5EED
+
+
+def hbm_peak_gbs():
+    if os.path.exists(PEAKS_FILE):
+        with open(PEAKS_FILE) as f:
+            v = json.load(f).get("hbm_gbs")
+        if v:
+            return float(v), "measured (MEASURED_PEAKS.json hbm_gbs, copy burst)"
+    return 6800.0, "fallback 6.8 TB/s"
+
+
+def measure_rht(kd, torch, layer, stream):
+    """Randomized-Hadamard rotation of the whole layer (Sec. 4, the Kashin-DCT+H
+    preprocessing): fp16 in, fp32 out, one kd_rht per matrix, timed with events on
+    the launch stream.  HBM-bound: 2 B read + 4 B written per parameter."""
+    outs = {}
+    for s, w in layer:
+        outs.setdefault(tuple(w.shape), torch.empty(tuple(w.shape), dtype=torch.float32, device=w.device))
+    evs = []
+    for rep in range(4):
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for s, w in layer:
+            kd.rht(w, RHT_SEED, out=outs[tuple(w.shape)], stream=stream)
+        b.record(stream)
+        if rep > 0:
+            evs.append((a, b))
+    torch.cuda.synchronize()
+    ms = sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+    params = sum(s.params for s, _ in layer)
+    nbytes = params * (2 + 4)
+    peak, basis = hbm_peak_gbs()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    del outs
+    return {"kernel": "rht_kernel (fp16 -> fp32, 7 launches per layer)", "ms_per_layer": round(ms, 4),
+            "params_per_s": round(params / (ms / 1e3), 1), "bound": "hbm", "achieved": round(gbs, 1),
+            "peak": peak, "unit": "GB/s", "frac": round(gbs / peak, 4), "peak_basis": basis,
+            "algorithmic_bytes_per_param": 6}
 
 
 def measure_refinement(kd, torch, layer, outs, wss, iters, stream, base_ms):
@@ -463,12 +507,19 @@ def run_profile_case(args) -> None:
     from paper_2609_11687_gb300 import kashin as kd
     spec = dataclasses.replace(synth.llama7b_layer(0)[args.profile_matrix], M=args.profile_m)
     w = synth.generate(spec, device="cuda")
+    if args.profile_kernel == "rht":
+        y = torch.empty(w.shape, dtype=torch.float32, device="cuda")
+        for _ in range(3):
+            kd.rht(w, RHT_SEED, out=y)
+        torch.cuda.synchronize()
+        log(f"[profile-case] ok: rht n={spec.N} m={spec.M}")
+        return
     ws = kd.Workspace(spec.N)
     out = None
     for _ in range(3):
-        out = kd.decompose(w, args.iters, spec.sign_seed, workspace=ws, out=out)
+        out = kd.decompose(w, args.iters, spec.sign_seed, workspace=ws, out=out, kmeans_iters=args.kmeans_iters)
     torch.cuda.synchronize()
-    log(f"[profile-case] ok: n={spec.N} m={spec.M} iters={args.iters}")
+    log(f"[profile-case] ok: n={spec.N} m={spec.M} iters={args.iters} kmeans={args.kmeans_iters}")
 
 
 def main():
@@ -486,6 +537,7 @@ def main():
     ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
     ap.add_argument("--profile-m", type=int, default=32768)
     ap.add_argument("--profile-matrix", type=int, default=0, help="layer matrix index (0 = q, 6 = down)")
+    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht"])
     args = ap.parse_args()
     if args.profile_case:
         run_profile_case(args)

@@ -155,6 +155,38 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v,
  * (KD_ERR_CUDA if the synchronisation fails). */
 kd_status kd_read_status(const void* workspace, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:
+ * the weights are rotated by a randomized Hadamard transform before the
+ * decomposition).  The paper does not give the construction; this library's:
+ *
+ *   forward   y_j = (I_{n/b} (x) H_b / sqrt(b)) diag(s) x_j
+ *   inverse   y_j = diag(s) (I_{n/b} (x) H_b / sqrt(b)) x_j       (the transpose)
+ *
+ * for every vector j, with H_b the Sylvester Hadamard matrix (H_1 = [1],
+ * H_2k = [[H_k, H_k], [H_k, -H_k]]) applied to each contiguous block of b
+ * entries, b = kd_rht_block(n) (the largest power of two dividing n, at most
+ * 16384), and s_i = -1 where bit 63 of SplitMix64(seed + (i+1)*0x9E3779B97F4A7C15)
+ * is set, +1 otherwise (the same generator as the decomposition's eps; give the
+ * rotation its own seed).
+ *
+ *   x        device, m vectors of n entries, vector j at x[j*ldx + i] (ldx >= n),
+ *            dtype KD_F32 / KD_F16 / KD_BF16.
+ *   y        device fp32, vector j at y[j*ldy + i] (ldy >= n).  y may be x itself
+ *            (in place) when dtype is KD_F32 and ldy == ldx; other overlaps are
+ *            the caller's error.
+ *   inverse  0 = forward, 1 = inverse.
+ *   stream   cudaStream_t as void*.
+ * Errors: KD_ERR_UNSUPPORTED_N unless n % 16 == 0 and 16 <= n <= 65536;
+ * KD_ERR_INVALID_ARG for m < 0, ld too small, bad dtype or flag, null pointers
+ * with m > 0, or an in-place call that is not fp32 with equal strides;
+ * KD_ERR_CUDA if the launch fails.  m == 0 enqueues nothing.  No workspace.
+ * To rotate along the other axis of a matrix (the output side of a two-sided
+ * rotation) pass its transpose. */
+int64_t kd_rht_block(int64_t n); /* block length b for vectors of length n, 0 if unsupported */
+kd_status kd_rht(const void* x, kd_dtype dtype, int64_t n, int64_t m, int64_t ldx, uint64_t seed, int inverse,
+                 float* y, int64_t ldy, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

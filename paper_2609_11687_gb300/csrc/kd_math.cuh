@@ -15,6 +15,14 @@
 
 namespace kd {
 
+// SplitMix64 output function (Steele, Lea & Flood, OOPSLA 2014): the sign of
+// entry j of a seeded sign set is bit 63 of mix(seed + (j + 1) * 0x9E3779B97F4A7C15).
+__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
 // ---------------------------------------------------------------------------
 // Compile-time cos / sin of 2*pi*a/b (double), from the Taylor series after an
 // exact rational reduction of the angle to [-pi/4, pi/4].

@@ -461,12 +461,6 @@ struct Xform {
 // rounded), the sign bits (SplitMix64 of seed + (j+1)*gamma, bit 63 set ->
 // eps_j = -1) and the cleared status word.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint64_t splitmix64_mix(uint64_t z) {
-  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
-  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
-  return z ^ (z >> 31);
-}
-
 __device__ __forceinline__ float2 root_w(long long m, long long b) {  // exp(-2 pi i m / b)
   double s, c;
   sincospi(2.0 * (double)m / (double)b, &s, &c);

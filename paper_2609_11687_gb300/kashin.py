@@ -30,7 +30,8 @@ KD_F32, KD_F16, KD_BF16 = 0, 1, 2
 KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
-           "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static")
+           "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
+           "kd_rht_block", "kd_rht")
 
 
 def _load() -> ctypes.CDLL:
@@ -59,6 +60,10 @@ def _load() -> ctypes.CDLL:
     lib.kd_reconstruct.restype = c_int
     lib.kd_read_status.argtypes = [c_vp, c_vp]
     lib.kd_read_status.restype = c_int
+    lib.kd_rht_block.argtypes = [c_i64]
+    lib.kd_rht_block.restype = c_i64
+    lib.kd_rht.argtypes = [c_vp, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_vp, c_i64, c_vp]
+    lib.kd_rht.restype = c_int
     return lib
 
 
@@ -120,6 +125,14 @@ def kd_reconstruct(codes_u, codes_v, centres_u, centres_v, n, m, sign_seed, out_
 
 def kd_read_status(workspace, stream) -> int:
     return lib.kd_read_status(workspace, stream)
+
+
+def kd_rht_block(n) -> int:
+    return int(lib.kd_rht_block(int(n)))
+
+
+def kd_rht(x, dtype, n, m, ldx, seed, inverse, y, ldy, stream) -> int:
+    return lib.kd_rht(x, dtype, n, m, ldx, ctypes.c_uint64(int(seed) & ((1 << 64) - 1)), inverse, y, ldy, stream)
 
 
 # ---------------------------------------------------------------------------
@@ -238,6 +251,24 @@ def apply_p(x, sign_seed: int, out=None, workspace: Optional[Workspace] = None, 
     st = kd_apply_p(x.data_ptr(), y.data_ptr(), n, m, sign_seed, ws.ptr, ws.nbytes, _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_apply_p")
+    return y
+
+
+def rht(x, seed: int, inverse: bool = False, out=None, stream=None):
+    """Randomized-Hadamard rotation of the rows of the (m, n) tensor ``x`` (fp32,
+    fp16 or bf16, unit inner stride) into an fp32 (m, n) tensor; ``out=x`` rotates
+    an fp32 tensor in place (Sec. 4, Kashin-DCT+H)."""
+    torch = _torch()
+    if x.dim() != 2 or x.stride(1) != 1:
+        raise ValueError("x must be a 2-D CUDA tensor with unit inner stride")
+    m, n = x.shape
+    y = out if out is not None else torch.empty((m, n), dtype=torch.float32, device=x.device)
+    if y.dtype != torch.float32 or y.shape != x.shape or y.stride(1) != 1:
+        raise ValueError("out must be an fp32 tensor of x's shape with unit inner stride")
+    st = kd_rht(x.data_ptr(), _dtype_code(x.dtype), n, m, x.stride(0), seed, 1 if inverse else 0, y.data_ptr(),
+                y.stride(0), _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_rht")
     return y
 
 
