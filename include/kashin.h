@@ -176,6 +176,11 @@ kd_status kd_read_status(const void* workspace, void* stream);
  *            (in place) when dtype is KD_F32 and ldy == ldx; other overlaps are
  *            the caller's error.
  *   inverse  0 = forward, 1 = inverse.
+ *   status   optional device word (NULL = none).  The kernel streams its input
+ *            through shared memory with bulk copies and bounds every wait for
+ *            one; if a copy has not landed after about a second it ORs
+ *            KD_RHT_ERR_TIMEOUT into *status, leaves that part of y unwritten
+ *            and returns.  The caller clears the word and reads it back.
  *   stream   cudaStream_t as void*.
  * Errors: KD_ERR_UNSUPPORTED_N unless n % 16 == 0 and 16 <= n <= 65536;
  * KD_ERR_INVALID_ARG for m < 0, ld too small, bad dtype or flag, null pointers
@@ -183,9 +188,10 @@ kd_status kd_read_status(const void* workspace, void* stream);
  * KD_ERR_CUDA if the launch fails.  m == 0 enqueues nothing.  No workspace.
  * To rotate along the other axis of a matrix (the output side of a two-sided
  * rotation) pass its transpose. */
+#define KD_RHT_ERR_TIMEOUT 1u
 int64_t kd_rht_block(int64_t n); /* block length b for vectors of length n, 0 if unsupported */
 kd_status kd_rht(const void* x, kd_dtype dtype, int64_t n, int64_t m, int64_t ldx, uint64_t seed, int inverse,
-                 float* y, int64_t ldy, void* stream);
+                 float* y, int64_t ldy, uint32_t* status, void* stream);
 
 #ifdef __cplusplus
 }

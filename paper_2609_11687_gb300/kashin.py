@@ -62,7 +62,7 @@ def _load() -> ctypes.CDLL:
     lib.kd_read_status.restype = c_int
     lib.kd_rht_block.argtypes = [c_i64]
     lib.kd_rht_block.restype = c_i64
-    lib.kd_rht.argtypes = [c_vp, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_vp, c_i64, c_vp]
+    lib.kd_rht.argtypes = [c_vp, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_vp, c_i64, c_vp, c_vp]
     lib.kd_rht.restype = c_int
     return lib
 
@@ -131,8 +131,9 @@ def kd_rht_block(n) -> int:
     return int(lib.kd_rht_block(int(n)))
 
 
-def kd_rht(x, dtype, n, m, ldx, seed, inverse, y, ldy, stream) -> int:
-    return lib.kd_rht(x, dtype, n, m, ldx, ctypes.c_uint64(int(seed) & ((1 << 64) - 1)), inverse, y, ldy, stream)
+def kd_rht(x, dtype, n, m, ldx, seed, inverse, y, ldy, status, stream) -> int:
+    return lib.kd_rht(x, dtype, n, m, ldx, ctypes.c_uint64(int(seed) & ((1 << 64) - 1)), inverse, y, ldy, status,
+                      stream)
 
 
 # ---------------------------------------------------------------------------
@@ -254,10 +255,11 @@ def apply_p(x, sign_seed: int, out=None, workspace: Optional[Workspace] = None, 
     return y
 
 
-def rht(x, seed: int, inverse: bool = False, out=None, stream=None):
+def rht(x, seed: int, inverse: bool = False, out=None, status=None, stream=None):
     """Randomized-Hadamard rotation of the rows of the (m, n) tensor ``x`` (fp32,
     fp16 or bf16, unit inner stride) into an fp32 (m, n) tensor; ``out=x`` rotates
-    an fp32 tensor in place (Sec. 4, Kashin-DCT+H)."""
+    an fp32 tensor in place (Sec. 4, Kashin-DCT+H).  ``status``: optional int32
+    device tensor of one element that collects KD_RHT_ERR_* bits."""
     torch = _torch()
     if x.dim() != 2 or x.stride(1) != 1:
         raise ValueError("x must be a 2-D CUDA tensor with unit inner stride")
@@ -266,7 +268,7 @@ def rht(x, seed: int, inverse: bool = False, out=None, stream=None):
     if y.dtype != torch.float32 or y.shape != x.shape or y.stride(1) != 1:
         raise ValueError("out must be an fp32 tensor of x's shape with unit inner stride")
     st = kd_rht(x.data_ptr(), _dtype_code(x.dtype), n, m, x.stride(0), seed, 1 if inverse else 0, y.data_ptr(),
-                y.stride(0), _stream(stream))
+                y.stride(0), status.data_ptr() if status is not None else None, _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_rht")
     return y

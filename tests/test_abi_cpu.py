@@ -107,18 +107,18 @@ def test_rht_block_and_validation(kd):
     for n in (0, 8, 24, 100, 65552, 131072):
         assert kd.kd_rht_block(n) == 0
     null = None
-    assert kd.kd_rht(1, 0, 100, 4, 100, 0, 0, 1, 100, null) == kd.KD_ERR_UNSUPPORTED_N
-    assert kd.kd_rht(1, 0, 256, -1, 256, 0, 0, 1, 256, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_rht(1, 0, 256, 4, 255, 0, 0, 1, 256, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_rht(1, 0, 256, 4, 256, 0, 0, 1, 255, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_rht(1, 9, 256, 4, 256, 0, 0, 1, 256, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_rht(1, 0, 256, 4, 256, 0, 2, 1, 256, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_rht(null, 0, 256, 4, 256, 0, 0, 1, 256, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(1, 0, 100, 4, 100, 0, 0, 1, 100, null, null) == kd.KD_ERR_UNSUPPORTED_N
+    assert kd.kd_rht(1, 0, 256, -1, 256, 0, 0, 1, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(1, 0, 256, 4, 255, 0, 0, 1, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(1, 0, 256, 4, 256, 0, 0, 1, 255, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(1, 9, 256, 4, 256, 0, 0, 1, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(1, 0, 256, 4, 256, 0, 2, 1, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(null, 0, 256, 4, 256, 0, 0, 1, 256, null, null) == kd.KD_ERR_INVALID_ARG
     # in place only for fp32 with equal strides
-    assert kd.kd_rht(4096, 1, 256, 4, 256, 0, 0, 4096, 256, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_rht(4096, 0, 256, 4, 256, 0, 0, 4096, 512, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(4096, 1, 256, 4, 256, 0, 0, 4096, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(4096, 0, 256, 4, 256, 0, 0, 4096, 512, null, null) == kd.KD_ERR_INVALID_ARG
     # nothing to do: no launch, no device needed
-    assert kd.kd_rht(null, 0, 256, 0, 256, 0, 0, null, 256, null) == kd.KD_OK
+    assert kd.kd_rht(null, 0, 256, 0, 256, 0, 0, null, 256, null, null) == kd.KD_OK
 
 
 def test_product_path_requires_library(tmp_path, monkeypatch):

@@ -28,6 +28,10 @@ def kd():
     return kashin
 
 
+def _status(torch):
+    return torch.zeros(1, dtype=torch.int32, device="cuda")
+
+
 def _check(y_dev, x_host, seed, inverse=False):
     ref = ko.randomized_hadamard(np.asarray(x_host, dtype=np.float64).T, seed, inverse=inverse).T
     y = y_dev.double().cpu().numpy()
@@ -43,11 +47,17 @@ def test_rht_forward_inverse_all_block_sizes(kd, n):
     g = torch.Generator().manual_seed(n)
     x = torch.randn((m, n), generator=g)
     seed = 1000 + n
-    y = kd.rht(x.cuda(), seed)
+    st = _status(torch)
+    y = kd.rht(x.cuda(), seed, status=st)
     torch.cuda.synchronize()
     _check(y, x.numpy(), seed)
-    z = kd.rht(y, seed, inverse=True)
+    z = kd.rht(y, seed, inverse=True, status=st)            # fp32 in: the staged path
+    zh = kd.rht(y.half(), seed, inverse=True, status=st)    # fp16 in, staged
+    yh = kd.rht(x.cuda().half(), seed, status=st)           # fp16 forward, staged
     torch.cuda.synchronize()
+    assert st.item() == 0
+    _check(zh, y.half().float().cpu().numpy(), seed, inverse=True)
+    _check(yh, x.half().float().numpy(), seed)
     _check(z, y.cpu().numpy(), seed, inverse=True)
     np.testing.assert_allclose(z.cpu().numpy(), x.numpy(), rtol=0, atol=4 * TOL * float(x.abs().max()))
 
@@ -60,6 +70,12 @@ def test_rht_half_inputs(kd, dtype):
     y = kd.rht(x.cuda(), 9)
     torch.cuda.synchronize()
     _check(y, x.float().numpy(), 9)
+    # strided rows (ld = 4096 + 64, still 16-byte aligned: staged, one copy per vector run)
+    base = torch.zeros((7, 4160), dtype=td)
+    base[:, :4096] = x
+    y2 = kd.rht(base.cuda()[:, :4096], 9)
+    torch.cuda.synchronize()
+    assert torch.equal(y2, y)
 
 
 def test_rht_strided_unaligned_inplace_and_empty(kd):
