@@ -54,10 +54,16 @@ def flops_per_vector(n: int, iters: int) -> float:
     return iters * (4 * 2 * n * math.log2(n) + 20 * n)
 
 
+# sources the N = 4096 decompose kernel is built from (the profile's DRAM figures
+# stay valid while these are unchanged)
+DECOMPOSE_SOURCES = ("kd_math.cuh", "kd_xform.cuh", "kd_kernels.cuh", "kd_plans.cuh", "kd_launch.cuh", "kd_ops.h",
+                     "kd_plan_4096.cu")
+
+
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_11687_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
+    for name in DECOMPOSE_SOURCES:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode())
             h.update(f.read())
@@ -284,6 +290,8 @@ def run_gpu(args) -> dict:
 
     # randomized-Hadamard pre-rotation (Kashin-DCT+H), HBM roofline
     rotation = measure_rht(kd, torch, layers[my_layers[-1]], stream)
+    # load-time inference expansion (App. C)
+    inference = measure_inference(kd, torch, layers[my_layers[-1]], iters, wss, stream)
 
     # end to end: pinned host input, H2D + decompose + D2H codes/centres each step
     e2e = None
@@ -308,6 +316,7 @@ def run_gpu(args) -> dict:
     if refinement is not None:
         result["kmeans_refinement"] = refinement
     result["hadamard_rotation"] = rotation
+    result["inference_load"] = inference
     if e2e is not None:
         result["e2e"] = e2e
     if rank == 0 and world == 1 and not args.skip_cpu:
@@ -329,6 +338,62 @@ def hbm_peak_gbs():
         if v:
             return float(v), "measured (MEASURED_PEAKS.json hbm_gbs, copy burst)"
     return 6800.0, "fallback 6.8 TB/s"
+
+
+def measure_inference(kd, torch, layer, iters, wss, stream):
+    """App. C at load time for one layer: dense W_hat = U_q + P V_q (kd_reconstruct,
+    fp16 out; one P per vector pair, ALU-bound) and the two expanded factor planes
+    for the folded product [X | XP][U_q; V_q] (kd_dequantise, fp16 out, HBM-bound)."""
+    decs = [(s, kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], stream=stream)) for s, w in layer]
+    outs = {}
+    for s, _ in layer:
+        outs.setdefault((s.M, s.N), torch.empty((s.M, s.N), dtype=torch.float16, device=layer[0][1].device))
+    def timed(fn, reps=4):
+        evs = []
+        for rep in range(reps):
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            if rep > 0:
+                evs.append((a, b))
+        torch.cuda.synchronize()
+        return sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+
+    def rec():
+        for s, d in decs:
+            kd.reconstruct(d, s.N, s.sign_seed, dtype=torch.float16, out=outs[(s.M, s.N)],
+                           workspace=wss[s.N], stream=stream)
+
+    def deq():
+        for s, d in decs:
+            o = outs[(s.M, s.N)]
+            kd.dequantise(d.codes_u, d.centres_u, s.N, out=o, stream=stream)
+            kd.dequantise(d.codes_v, d.centres_v, s.N, out=o, stream=stream)
+
+    ms_rec = timed(rec)
+    ms_deq = timed(deq)
+    params = sum(s.params for s, _ in layer)
+    # one P (a DCT and an inverse DCT) per vector: 2 * 2 n log2 n flops, plus n adds
+    import math
+    flops = sum(s.M * (4 * s.N * math.log2(s.N) + s.N) for s, _ in layer)
+    peak_alu = SM_COUNT * FP32_LANES_PER_SM * 2 * 2.070e9 / 1e12
+    deq_bytes = 2 * params * (0.25 + 2)
+    hbm, basis = hbm_peak_gbs()
+    del outs, decs
+    return {
+        "reconstruct": {"kernel": "reconstruct_kernel (codes -> fp16 W_hat, 7 launches per layer)",
+                        "ms_per_layer": round(ms_rec, 4), "params_per_s": round(params / (ms_rec / 1e3), 1),
+                        "bound": "alu", "achieved": round(flops / (ms_rec / 1e3) / 1e12, 3),
+                        "peak": round(peak_alu, 2), "unit": "TFLOP/s",
+                        "frac": round(flops / (ms_rec / 1e3) / 1e12 / peak_alu, 4)},
+        "dequantise": {"kernel": "dequant_rows_kernel (both planes -> fp16, 14 launches per layer)",
+                       "ms_per_layer": round(ms_deq, 4), "bound": "hbm",
+                       "achieved": round(deq_bytes / (ms_deq / 1e3) / 1e9, 1), "peak": hbm, "unit": "GB/s",
+                       "frac": round(deq_bytes / (ms_deq / 1e3) / 1e9 / hbm, 4), "peak_basis": basis,
+                       "algorithmic_bytes_per_param": 4.5},
+    }
 
 
 def measure_rht(kd, torch, layer, stream):

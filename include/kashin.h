@@ -144,7 +144,8 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
 
 /* Dense re-materialisation W_hat = U_q + P V_q (App. C): vector j of w_hat is
  * centres_u[j][code_u] + P(centres_v[j][code_v]).  Inputs as produced by
- * kd_decompose; output dtype out_dtype in `layout` with leading dimension ld. */
+ * kd_decompose (centres 16-byte aligned, KD_ERR_INVALID_ARG otherwise); output dtype
+ * out_dtype in `layout` with leading dimension ld. */
 kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v,
                          const float* centres_u, const float* centres_v, int64_t n, int64_t m,
                          uint64_t sign_seed, kd_dtype out_dtype, kd_layout layout, void* w_hat,
@@ -154,6 +155,20 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v,
  * by the last kd_decompose on this workspace held a NaN or Inf, KD_OK otherwise
  * (KD_ERR_CUDA if the synchronisation fails). */
 kd_status kd_read_status(const void* workspace, void* stream);
+
+/* Dequantise one 2-bit factor plane (App. C, inference): out entry i of vector j =
+ * centres[j*4 + code_j(i)], code_j(i) = bits 2(i%16)..2(i%16)+1 of codes[j*ceil(n/16) + i/16].
+ * With U_q and V_q expanded this way the layer product folds as
+ *   X W = X U_q + (X P) V_q = [X | XP] [U_q; V_q]      (App. C, Eq. inference_factor),
+ * XP from kd_apply_p on the rows of X; kd_reconstruct gives W_hat = U_q + P V_q itself.
+ *   codes    device, m x ceil(n/16) uint32 (kd_decompose's codes_u or codes_v).
+ *   centres  device, m x 4 fp32 ascending (centres_u or centres_v), 16-byte aligned.
+ *   out      device, dtype out_dtype, layout as for kd_decompose's input (ld >= n for
+ *            KD_VEC_ROWS, >= m for KD_VEC_COLUMNS).
+ * No workspace.  Errors: KD_ERR_INVALID_ARG (sizes, enums, ld, null or unaligned
+ * pointers with m > 0), KD_ERR_CUDA (launch).  m == 0 enqueues nothing. */
+kd_status kd_dequantise(const uint32_t* codes, const float* centres, int64_t n, int64_t m, kd_dtype out_dtype,
+                        kd_layout layout, void* out, int64_t ld, void* stream);
 
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:

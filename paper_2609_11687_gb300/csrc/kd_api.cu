@@ -217,6 +217,8 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
   if (!ops) return KD_ERR_UNSUPPORTED_N;
   if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
   if (m > 0 && (!codes_u || !codes_v || !centres_u || !centres_v || !w_hat)) return KD_ERR_INVALID_ARG;
+  if (m > 0 && ((reinterpret_cast<uintptr_t>(centres_u) | reinterpret_cast<uintptr_t>(centres_v)) % 16 != 0))
+    return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
   if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;

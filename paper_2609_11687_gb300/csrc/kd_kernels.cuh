@@ -656,32 +656,51 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
     const int64_t colA = 2 * pr;
     const bool hasB = (colA + 1) < p.m;
     const int64_t colB = hasB ? colA + 1 : colA;
+    // the four centre sets of the pair (the same for the whole team: broadcast loads)
+    const float4 cuA = __ldg(reinterpret_cast<const float4*>(p.centres_u) + colA);
+    const float4 cuB = __ldg(reinterpret_cast<const float4*>(p.centres_u) + colB);
+    const float4 cvA = __ldg(reinterpret_cast<const float4*>(p.centres_v) + colA);
+    const float4 cvB = __ldg(reinterpret_cast<const float4*>(p.centres_v) + colB);
+    auto pick = [](const float4& c, uint32_t q) -> float {
+      const float lo = (q & 1u) ? c.y : c.x;
+      const float hi = (q & 1u) ? c.w : c.z;
+      return (q & 2u) ? hi : lo;
+    };
+    // code words of the pair staged in shared memory, word w as (uA, uB, vA, vB)
+    uint4* cw = reinterpret_cast<uint4*>(buf);
+    for (int w = lt; w < WPV; w += T) {
+      cw[w] = make_uint4(__ldg(&p.codes_u[colA * WPV + w]), __ldg(&p.codes_u[colB * WPV + w]),
+                         __ldg(&p.codes_v[colA * WPV + w]), __ldg(&p.codes_v[colB * WPV + w]));
+    }
+    team_sync<PL>();
     float2 uq[E], vq[E];
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
-      const int word = nat >> 4, sh = 2 * (nat & 15);
-      const int cuA = (__ldg(&p.codes_u[colA * WPV + word]) >> sh) & 3;
-      const int cvA = (__ldg(&p.codes_v[colA * WPV + word]) >> sh) & 3;
-      float ua = __ldg(&p.centres_u[colA * 4 + cuA]);
-      float va = __ldg(&p.centres_v[colA * 4 + cvA]);
-      float ub = 0.f, vb = 0.f;
-      if (hasB) {
-        const int cuB = (__ldg(&p.codes_u[colB * WPV + word]) >> sh) & 3;
-        const int cvB = (__ldg(&p.codes_v[colB * WPV + word]) >> sh) & 3;
-        ub = __ldg(&p.centres_u[colB * 4 + cuB]);
-        vb = __ldg(&p.centres_v[colB * 4 + cvB]);
-      }
-      uq[j] = make_float2(ua, ub);
-      vq[j] = make_float2(va, vb);
+      const uint4 c = cw[nat >> 4];
+      const int sh = 2 * (nat & 15);
+      uq[j] = make_float2(pick(cuA, (c.x >> sh) & 3u), pick(cuB, (c.y >> sh) & 3u));
+      vq[j] = make_float2(pick(cvA, (c.z >> sh) & 3u), pick(cvB, (c.w >> sh) & 3u));
     }
+    team_sync<PL>();  // the transform reuses buf
     xf.apply(vq);
-    if (active) {
+    // W_hat = U_q + P V_q, staged in natural order so the stores are contiguous
+    team_sync<PL>();
 #pragma unroll
-      for (int j = 0; j < E; ++j) {
-        const int nat = nat_of<N>(lt + j * T);
-        store_elem(p.out, p.dtype, elem_index(p.layout, colA, nat, p.ld), __fadd_rn(uq[j].x, vq[j].x));
-        if (hasB) store_elem(p.out, p.dtype, elem_index(p.layout, colB, nat, p.ld), __fadd_rn(uq[j].y, vq[j].y));
+    for (int j = 0; j < E; ++j) {
+      const int nat = nat_of<N>(lt + j * T);
+      buf[nat] = make_float2(__fadd_rn(uq[j].x, vq[j].x), __fadd_rn(uq[j].y, vq[j].y));
+    }
+    team_sync<PL>();
+    if (active) {
+      for (int i = 2 * lt; i < N; i += 2 * T) {
+        const float2 e0 = buf[i], e1 = buf[i + 1];   // entries i, i + 1 of (A, B)
+        store_elem(p.out, p.dtype, elem_index(p.layout, colA, i, p.ld), e0.x);
+        store_elem(p.out, p.dtype, elem_index(p.layout, colA, i + 1, p.ld), e1.x);
+        if (hasB) {
+          store_elem(p.out, p.dtype, elem_index(p.layout, colB, i, p.ld), e0.y);
+          store_elem(p.out, p.dtype, elem_index(p.layout, colB, i + 1, p.ld), e1.y);
+        }
       }
     }
     team_sync<PL>();

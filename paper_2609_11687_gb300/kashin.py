@@ -31,7 +31,7 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
-           "kd_rht_block", "kd_rht")
+           "kd_rht_block", "kd_rht", "kd_dequantise")
 
 
 def _load() -> ctypes.CDLL:
@@ -60,6 +60,8 @@ def _load() -> ctypes.CDLL:
     lib.kd_reconstruct.restype = c_int
     lib.kd_read_status.argtypes = [c_vp, c_vp]
     lib.kd_read_status.restype = c_int
+    lib.kd_dequantise.argtypes = [c_vp, c_vp, c_i64, c_i64, c_int, c_int, c_vp, c_i64, c_vp]
+    lib.kd_dequantise.restype = c_int
     lib.kd_rht_block.argtypes = [c_i64]
     lib.kd_rht_block.restype = c_i64
     lib.kd_rht.argtypes = [c_vp, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_vp, c_i64, c_vp, c_vp]
@@ -125,6 +127,10 @@ def kd_reconstruct(codes_u, codes_v, centres_u, centres_v, n, m, sign_seed, out_
 
 def kd_read_status(workspace, stream) -> int:
     return lib.kd_read_status(workspace, stream)
+
+
+def kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream) -> int:
+    return lib.kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream)
 
 
 def kd_rht_block(n) -> int:
@@ -253,6 +259,22 @@ def apply_p(x, sign_seed: int, out=None, workspace: Optional[Workspace] = None, 
     if st != KD_OK:
         raise KashinError(st, "kd_apply_p")
     return y
+
+
+def dequantise(codes, centres, n: int, dtype=None, layout: str = "rows", out=None, stream=None):
+    """Dense factor matrix from one 2-bit code plane and its centres (App. C):
+    (m, n) for layout "rows", (n, m) for "columns"."""
+    torch = _torch()
+    dtype = dtype or torch.float32
+    m = codes.shape[0]
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    if out is None:
+        out = torch.empty((m, n) if lay == KD_VEC_ROWS else (n, m), dtype=dtype, device=codes.device)
+    st = kd_dequantise(codes.data_ptr(), centres.data_ptr(), n, m, _dtype_code(out.dtype), lay, out.data_ptr(),
+                       out.stride(0), _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_dequantise")
+    return out
 
 
 def rht(x, seed: int, inverse: bool = False, out=None, status=None, stream=None):

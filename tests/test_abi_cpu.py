@@ -121,6 +121,18 @@ def test_rht_block_and_validation(kd):
     assert kd.kd_rht(null, 0, 256, 0, 256, 0, 0, null, 256, null, null) == kd.KD_OK
 
 
+def test_dequantise_validation(kd):
+    null = None
+    assert kd.kd_dequantise(16, 16, 0, 4, 0, 0, 16, 16, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise(16, 16, 64, 4, 5, 0, 16, 64, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise(16, 16, 64, 4, 0, 3, 16, 64, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise(16, 16, 64, 4, 0, 0, 16, 63, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise(16, 16, 64, 4, 0, 1, 16, 3, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise(null, 16, 64, 4, 0, 0, 16, 64, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise(16, 8, 64, 4, 0, 0, 16, 64, null) == kd.KD_ERR_INVALID_ARG   # centres unaligned
+    assert kd.kd_dequantise(null, null, 64, 0, 0, 0, null, 64, null) == kd.KD_OK
+
+
 def test_product_path_requires_library(tmp_path, monkeypatch):
     """Importing the binding without the built library raises: no CPU fallback."""
     import importlib.util
