@@ -232,10 +232,8 @@ struct DftPrime {
         constexpr int NN = decltype(nn)::value;
         constexpr float c = (float)cos2pi((long long)NN * K, R);
         constexpr float s = (float)sin2pi((long long)NN * K, R);
-        ak.x = __fmaf_rn(a[NN].x, c, ak.x);
-        ak.y = __fmaf_rn(a[NN].y, c, ak.y);
-        bk.x = __fmaf_rn(b[NN].x, s, bk.x);
-        bk.y = __fmaf_rn(b[NN].y, s, bk.y);
+        ak = __ffma2_rn(a[NN], make_float2(c, c), ak);
+        bk = __ffma2_rn(b[NN], make_float2(s, s), bk);
       });
       // forward: X_k = ak - i bk, X_{R-k} = ak + i bk ; inverse: the reverse
       if constexpr (DIR < 0) {
@@ -275,10 +273,9 @@ __device__ __forceinline__ void dft_prime_stream(Load&& load, Store&& store) {
       constexpr int NN = decltype(nn)::value;
       constexpr float c = (float)cos2pi((long long)NN * K, R);
       constexpr float sn = (float)sin2pi((long long)NN * K, R);
-      ak.x = __fmaf_rn(a[NN].x, c, ak.x);
-      ak.y = __fmaf_rn(a[NN].y, c, ak.y);
-      bk.x = __fmaf_rn(b[NN].x, sn, bk.x);
-      bk.y = __fmaf_rn(b[NN].y, sn, bk.y);
+      // one packed FMA per complex term (both lanes round exactly like two FFMAs)
+      ak = __ffma2_rn(a[NN], make_float2(c, c), ak);
+      bk = __ffma2_rn(b[NN], make_float2(sn, sn), bk);
     });
     if constexpr (DIR < 0) {
       store(ic<K>{}, sub_ib(ak, bk));
