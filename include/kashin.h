@@ -203,6 +203,11 @@ kd_status kd_dequantise(const uint32_t* codes, const float* centres, int64_t n, 
  * KD_ERR_CUDA if the launch fails.  m == 0 enqueues nothing.  No workspace.
  * To rotate along the other axis of a matrix (the output side of a two-sided
  * rotation) pass its transpose. */
+/* Measured FP32 throughput of the current device in TFLOP/s (packed FFMA2 chains on
+ * every SM, best of three timed launches on `stream`; synchronises the stream).
+ * Used as the measured denominator of the transform kernels' ALU roofline. */
+kd_status kd_measure_fp32_peak(double* tflops, void* stream);
+
 #define KD_RHT_ERR_TIMEOUT 1u
 int64_t kd_rht_block(int64_t n); /* block length b for vectors of length n, 0 if unsupported */
 kd_status kd_rht(const void* x, kd_dtype dtype, int64_t n, int64_t m, int64_t ldx, uint64_t seed, int inverse,

@@ -31,7 +31,7 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
-           "kd_rht_block", "kd_rht", "kd_dequantise")
+           "kd_rht_block", "kd_rht", "kd_dequantise", "kd_measure_fp32_peak")
 
 
 def _load() -> ctypes.CDLL:
@@ -60,6 +60,8 @@ def _load() -> ctypes.CDLL:
     lib.kd_reconstruct.restype = c_int
     lib.kd_read_status.argtypes = [c_vp, c_vp]
     lib.kd_read_status.restype = c_int
+    lib.kd_measure_fp32_peak.argtypes = [c_vp, c_vp]
+    lib.kd_measure_fp32_peak.restype = c_int
     lib.kd_dequantise.argtypes = [c_vp, c_vp, c_i64, c_i64, c_int, c_int, c_vp, c_i64, c_vp]
     lib.kd_dequantise.restype = c_int
     lib.kd_rht_block.argtypes = [c_i64]
@@ -131,6 +133,15 @@ def kd_read_status(workspace, stream) -> int:
 
 def kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream) -> int:
     return lib.kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream)
+
+
+def measure_fp32_peak(stream=None) -> float:
+    """Measured FP32 TFLOP/s of the current device (packed FFMA chains)."""
+    out = ctypes.c_double(0.0)
+    st = lib.kd_measure_fp32_peak(ctypes.byref(out), _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_measure_fp32_peak")
+    return out.value
 
 
 def kd_rht_block(n) -> int:
