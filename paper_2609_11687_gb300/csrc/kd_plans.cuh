@@ -21,7 +21,9 @@ using Plan2048 = Plan<2048, 128, 1, USMEM, 4, 16, 16, 8>;
 using Plan3072 = Plan<3072, 192, 1, USMEM, 2, 16, 12, 16>;
 using Plan4096 = Plan<4096, 256, 1, USMEM, 2, 16, 16, 16>;
 using Plan8192 = Plan<8192, 512, 1, USMEM, 1, 16, 32, 16>;
-using Plan11008 = Plan<11008, 256, 1, UGMEM, 1, 43, 16, 16>;
+// u (88 KB) in shared memory; the twiddle table then no longer fits beside it and
+// is read through L1/L2
+using Plan11008 = Plan<11008, 256, 1, USMEM, 1, 43, 16, 16>;
 using Plan14336 = Plan<14336, 512, 1, UGMEM, 1, 28, 16, 32>;
 using Plan16384 = Plan<16384, 512, 1, UGMEM, 1, 32, 32, 16>;
 }  // namespace kd
