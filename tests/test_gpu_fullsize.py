@@ -42,14 +42,17 @@ def kd():
     return kashin
 
 
-@pytest.mark.parametrize("cfg,spec", CASES, ids=[f"{c}-{s.name}" for c, s in CASES])
-def test_fullsize_sampled_parity(kd, cfg, spec):
+# the k-means refinement at full size too: the gate and down projections of the 7B layer
+KM_CASES = [("cfg3-km3", s) for s in synth.config3() if s.name.endswith(("gate", "down"))]
+
+
+def _run(kd, cfg, spec, kmeans_iters=0):
     import torch
     w = synth.generate(spec, device="cuda")                  # (M, N) fp16, device generator
-    full = kd.decompose(w, ITERS, spec.sign_seed, coeffs=True)
+    full = kd.decompose(w, ITERS, spec.sign_seed, coeffs=True, kmeans_iters=kmeans_iters)
     idx = synth.pair_aligned_sample(spec.M, SAMPLE_VECTORS, seed=spec.seed + 17)
     sub = w[idx].contiguous()
-    dev = parity.device_outputs(kd, sub, ITERS, spec.sign_seed, trace=True)
+    dev = parity.device_outputs(kd, sub, ITERS, spec.sign_seed, trace=True, kmeans_iters=kmeans_iters)
     torch.cuda.synchronize()
     sel = torch.tensor(idx, device="cuda")
     for name in ("centres_u", "centres_v", "coeffs"):
@@ -57,6 +60,16 @@ def test_fullsize_sampled_parity(kd, cfg, spec):
     np.testing.assert_array_equal(full.codes_u[sel].cpu().numpy(), dev["words_u"])
     np.testing.assert_array_equal(full.codes_v[sel].cpu().numpy(), dev["words_v"])
     x = sub.double().cpu().numpy().T
-    rep = parity.compare(x, spec.sign_seed, ITERS, dev)
+    rep = parity.compare(x, spec.sign_seed, ITERS, dev, kmeans_iters=kmeans_iters)
     print(cfg, spec.name, rep)
     rep.check()
+
+
+@pytest.mark.parametrize("cfg,spec", CASES, ids=[f"{c}-{s.name}" for c, s in CASES])
+def test_fullsize_sampled_parity(kd, cfg, spec):
+    _run(kd, cfg, spec)
+
+
+@pytest.mark.parametrize("cfg,spec", KM_CASES, ids=[f"{c}-{s.name}" for c, s in KM_CASES])
+def test_fullsize_sampled_parity_kmeans(kd, cfg, spec):
+    _run(kd, cfg, spec, kmeans_iters=3)
