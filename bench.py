@@ -9,13 +9,20 @@ fp16), so no step re-reads an input another step touched; every input is larger
 than L2.
 
 Prints ONE JSON line on rank 0.  Extras in that line:
-  roofline      ALU roofline of the dominant kernel (decompose, N = 4096), measured
-                with CUDA events on the launch stream inside the timed region.
-  cpu_baseline  the CPU oracle (fp64, dense DCT matrix) on a bounded sample.
-  e2e           same metric with host (pinned) input buffers, H2D + D2H in the loop.
-  clocks        nvidia-smi samples taken during the timed region.
+  roofline           ALU roofline of the dominant kernel (decompose at the length
+                     carrying most parameters; N = 4096 for the 7B layer), measured
+                     with CUDA events on the launch stream inside the timed region,
+                     plus a measured FP32 peak and the FFT-count figure.
+  cpu_baseline       the CPU oracle (fp64, dense DCT matrix) on a bounded sample.
+  e2e                same metric with host (pinned) input buffers, H2D + D2H in the loop.
+  clocks             nvidia-smi samples taken during the timed region.
+  kmeans_refinement  cost of 3 Lloyd iterations of the centres (Sec. 2.1).
+  hadamard_rotation  the Kashin-DCT+H pre-rotation of the layer, HBM roofline.
+  inference_load     W_hat re-materialisation and factor expansion (App. C).
 
-``--impl reference`` times the CPU oracle instead (the reference arm).
+``--workload`` picks another synthetic stand-in per step (OPT-125M, Pythia-6.9B and
+Mistral-7B-shaped layers, the single 256x256 matrix); ``--impl reference`` times the
+CPU oracle instead (the reference arm).
 """
 
 from __future__ import annotations
@@ -37,10 +44,40 @@ if ROOT not in sys.path:
 METRIC = "params decomposed+2-bit coded/sec at 7B layer shapes; % of roofline"
 UNIT = "params/s"
 ITERS = 16
-LAYERS = 32
 PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 PROFILE_FILE = os.path.join(ROOT, "profiles", "decompose_n4096_llama7b.json")
+
+
+def _workloads():
+    """Per-step workloads: name -> (number of seeded layers cycled, layer(L) -> specs,
+    description).  The default is the Llama-2-7B layer; the others are the remaining
+    synthetic stand-ins of the paper's models, for their own throughput lines."""
+    from paper_2609_11687_gb300 import synth
+
+    def fam(name):
+        return lambda L: [s for s in synth.config5([L]) if s.name.startswith(name)]
+
+    return {
+        "llama7b": (32, synth.llama7b_layer,
+                    "llama2-7b decoder layer per step: q,k,v,o 4096x4096, gate,up 4096x11008, down 11008x4096 "
+                    "(202,375,168 params, fp16 Student-t nu=4 std 0.015, 0.1% input channels x20), cycling the "
+                    "32 seeded layers of the 7B stack resident in HBM"),
+        "w256": (1, lambda L: synth.config1(),
+                 "one 256x256 fp32 matrix per step, 0.02 N(0,1), seed 0 (65,536 params)"),
+        "opt125m": (12, lambda L: synth.config2([L]),
+                    "OPT-125M-shaped layer per step: q,k,v,o 768x768, fc1 768x3072, fc2 3072x768 (7,077,888 "
+                    "params, fp16 Student-t nu=4 std 0.02), cycling 12 seeded layers"),
+        "pythia6.9b": (32, fam("pythia"),
+                       "Pythia-6.9B-like layer per step: qkv 4096x12288, dense 4096x4096, h->4h 4096x16384, "
+                       "4h->h 16384x4096 (201,326,592 params, fp16 Student-t nu=3 std 0.02, 0.05% entries x50), "
+                       "cycling 32 seeded layers"),
+        "mistral7b": (32, fam("mistral"),
+                      "Mistral-7B-like layer per step: q,o 4096x4096, k,v 4096x1024, gate,up 4096x14336, down "
+                      "14336x4096 (218,103,808 params, fp16 Student-t nu=3 std 0.02, 0.05% entries x50), cycling "
+                      "32 seeded layers"),
+    }
 SM_COUNT = 152
+L2_BYTES = 129 * 1024 * 1024
 FP32_LANES_PER_SM = 128
 
 
@@ -206,49 +243,71 @@ def run_gpu(args) -> dict:
     # this rank's layers: rank, rank + world, ...  (weak scaling, no data exchange)
     steps_total = args.warmup + args.steps
     from paper_2609_11687_gb300 import shard
-    my_layers = shard.layer_schedule(rank, world, steps_total, LAYERS)
+    n_layers, layer_fn, workload_desc = _workloads()[args.workload]
+    my_layers = shard.layer_schedule(rank, world, steps_total, n_layers)
     uniq = sorted(set(my_layers))
-    log(f"[bench] rank {rank}/{world}: generating {len(uniq)} Llama-2-7B-shaped layers on {dev}")
+    log(f"[bench] rank {rank}/{world}: generating {len(uniq)} {args.workload} layers on {dev}")
     t0 = time.time()
     layers = {}
     for L in uniq:
-        specs = synth.llama7b_layer(L)
+        specs = layer_fn(L)
         layers[L] = [(s, synth.generate(s, device=dev)) for s in specs]
     torch.cuda.synchronize()
     log(f"[bench] generated in {time.time() - t0:.1f}s")
-    layer_params = synth.total_params(synth.llama7b_layer(0))
+    layer_params = synth.total_params(layer_fn(0))
+    # the dominant kernel: the vector length carrying most of the parameters
+    by_n = {}
+    for s_ in layer_fn(0):
+        by_n[s_.N] = by_n.get(s_.N, 0) + s_.params
+    NDOM = max(by_n, key=by_n.get)
 
-    # outputs and workspaces, allocated once
-    outs = {}
-    wss = {}
-    for s, w in layers[uniq[0]]:
-        key = (s.N, s.M)
-        if key not in outs:
-            words = (s.N + 15) // 16
-            outs[key] = kd.Decomposed(
-                codes_u=torch.empty((s.M, words), dtype=torch.int32, device=dev),
-                codes_v=torch.empty((s.M, words), dtype=torch.int32, device=dev),
-                centres_u=torch.empty((s.M, 4), dtype=torch.float32, device=dev),
-                centres_v=torch.empty((s.M, 4), dtype=torch.float32, device=dev),
-                coeffs=None, u=None, vhat=None, resid=None, trace=None)
-        if s.N not in wss:
-            wss[s.N] = kd.Workspace(s.N, dev)
+    # outputs (one set per matrix of the layer) and workspaces, allocated once
+    layer0 = layers[uniq[0]]
+    outs = []
+    for s, w in layer0:
+        words = (s.N + 15) // 16
+        outs.append(kd.Decomposed(
+            codes_u=torch.empty((s.M, words), dtype=torch.int32, device=dev),
+            codes_v=torch.empty((s.M, words), dtype=torch.int32, device=dev),
+            centres_u=torch.empty((s.M, 4), dtype=torch.float32, device=dev),
+            centres_v=torch.empty((s.M, 4), dtype=torch.float32, device=dev),
+            coeffs=None, u=None, vhat=None, resid=None, trace=None))
+    # matrices of one vector length go out in one kd_decompose_batch launch
+    groups = {}
+    for i, (s, _) in enumerate(layer0):
+        groups.setdefault(s.N, []).append(i)
+    wss = {n_: kd.Workspace(n_, dev) for n_ in groups}
+    wsb = {n_: kd.Workspace(n_, dev, count=len(ix)) for n_, ix in groups.items()}
     stream = torch.cuda.current_stream()
 
-    ev_main = {}  # per-launch events of the dominant kernel (N = 4096)
+    # kernels per step: batch = set-up + sign sets + decompose per length; single =
+    # set-up + decompose per matrix (longer lengths always run one launch per matrix)
+    if args.launch == "batch":
+        launches_per_step = sum((3 if len(ix) > 1 else 2) if kd.kd_batchable(n_) else 2 * len(ix)
+                                for n_, ix in groups.items())
+    else:
+        launches_per_step = 2 * len(layer0)
+    ev_main = {}  # per-launch events of the dominant kernel
 
     def run_layer(L, record=False):
-        for s, w in layers[L]:
-            o = outs[(s.N, s.M)]
-            if record and s.N == 4096:
+        mats = layers[L]
+        for n_, ix in groups.items():
+            rec = record and n_ == NDOM
+            if rec:
                 e0 = torch.cuda.Event(enable_timing=True)
                 e1 = torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-            kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream,
-                         kmeans_iters=args.kmeans_iters)
-            if record and s.N == 4096:
+            if args.launch == "batch":
+                kd.decompose_batch([mats[i][1] for i in ix], iters, [mats[i][0].sign_seed for i in ix],
+                                   workspace=wsb[n_], outs=[outs[i] for i in ix], stream=stream,
+                                   kmeans_iters=args.kmeans_iters)
+            else:
+                for i in ix:
+                    kd.decompose(mats[i][1], iters, mats[i][0].sign_seed, workspace=wss[n_], out=outs[i],
+                                 stream=stream, kmeans_iters=args.kmeans_iters)
+            if rec:
                 e1.record(stream)
-                ev_main.setdefault("ev", []).append((e0, e1, s.M))
+                ev_main.setdefault("ev", []).append((e0, e1, sum(mats[i][0].M for i in ix)))
 
     for i in range(args.warmup):
         run_layer(my_layers[i])
@@ -263,33 +322,53 @@ def run_gpu(args) -> dict:
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
-    start.record(stream)
-    for i in range(args.steps):
-        run_layer(my_layers[args.warmup + i], record=True)
-    end.record(stream)
+    step_bytes = sum(w.numel() * w.element_size() for _, w in layers[uniq[0]])
+    flush = None
+    if step_bytes < 2 * L2_BYTES:
+        # a step's input fits in L2: time each step alone and overwrite L2 between steps
+        flush = torch.empty(4 * L2_BYTES // 4, dtype=torch.float32, device=dev)
+        step_ms = 0.0
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            run_layer(my_layers[args.warmup + i], record=True)
+            b.record(stream)
+            b.synchronize()
+            step_ms += a.elapsed_time(b)
+        l2_note = f"L2 overwritten between timed steps ({4 * L2_BYTES >> 20} MB write); steps timed one by one"
+    else:
+        start.record(stream)
+        for i in range(args.steps):
+            run_layer(my_layers[args.warmup + i], record=True)
+        end.record(stream)
+        l2_note = f"inputs larger than L2 ({step_bytes / 1e6:.0f} MB per step, distinct layer every step)"
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     clk = clocks.stop()
-    elapsed_ms, total_params = shard.aggregate(start.elapsed_time(end), args.steps * layer_params)
+    elapsed_ms, total_params = shard.aggregate(step_ms if flush is not None else start.elapsed_time(end),
+                                               args.steps * layer_params)
     value = total_params / (elapsed_ms / 1e3)
+    del flush
 
     # dominant kernel: average launch duration over the timed region
     launches = ev_main.get("ev", [])
     dur = sum(a.elapsed_time(b) for a, b, _ in launches) / max(1, len(launches))
     vec_per_launch = sum(mm for _, _, mm in launches) / max(1, len(launches))
-    fl = flops_per_vector(4096, iters) * vec_per_launch
+    fl = flops_per_vector(NDOM, iters) * vec_per_launch
     achieved_tflops = fl / (dur / 1e3) / 1e12
     peak = SM_COUNT * FP32_LANES_PER_SM * 2 * 2.070e9 / 1e12
     traffic = None
     if os.path.exists(PROFILE_FILE):
         with open(PROFILE_FILE) as f:
             prof = json.load(f)
-        if prof.get("kernel_hash") == kernel_source_hash() and prof.get("iters") == iters:
+        if prof.get("kernel_hash") == kernel_source_hash() and prof.get("iters") == iters and NDOM == 4096:
             traffic = prof["dram_bytes_per_vector"] * vec_per_launch
     roofline = {"bound": "alu", "achieved": round(achieved_tflops, 3), "peak": round(peak, 2),
                 "unit": "TFLOP/s", "frac": round(achieved_tflops / peak, 4), "traffic": traffic,
-                "kernel": "decompose_kernel<N=4096>", "launch_ms": round(dur, 3),
+                "kernel": f"decompose_kernel<N={NDOM}>", "launch_ms": round(dur, 3),
                 "peak_basis": "FP32 FMA: 152 SMs x 128 lanes x 2 flop x 2070 MHz (max clock)"}
     if clk.get("sm_mhz"):
         roofline["frac_at_measured_clock"] = round(achieved_tflops / (peak * clk["sm_mhz"] / 2070.0), 4)
@@ -298,14 +377,14 @@ def run_gpu(args) -> dict:
     meas = kd.measure_fp32_peak(stream)
     roofline["measured_fp32_peak"] = round(meas, 2)
     roofline["frac_of_measured_fp32_peak"] = round(achieved_tflops / meas, 4)
-    fl_fft = fft_flops_per_vector(4096, iters) * vec_per_launch
+    fl_fft = fft_flops_per_vector(NDOM, iters) * vec_per_launch
     roofline["achieved_fft_count"] = round(fl_fft / (dur / 1e3) / 1e12, 3)
 
     # k-means refinement (Sec. 2.1): cost of KM_PROBE Lloyd iterations on the dominant
     # kernel, timed on the same matrices right after the timed region
     refinement = None
     if args.kmeans_iters == 0:
-        refinement = measure_refinement(kd, torch, layers[my_layers[-1]], outs, wss, iters, stream, dur)
+        refinement = measure_refinement(kd, torch, layers[my_layers[-1]], outs, wss, iters, stream, NDOM)
 
     # randomized-Hadamard pre-rotation (Kashin-DCT+H), HBM roofline
     rotation = measure_rht(kd, torch, layers[my_layers[-1]], stream)
@@ -321,15 +400,13 @@ def run_gpu(args) -> dict:
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(elapsed_ms / args.steps, 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": "llama2-7b decoder layer per step: q,k,v,o 4096x4096, gate,up 4096x11008, "
-                               "down 11008x4096 (202,375,168 params, fp16 Student-t nu=4 std 0.015, 0.1% input "
-                               "channels x20), cycling the 32 seeded layers of the 7B stack resident in HBM",
+        "config": {"workload": workload_desc, "launch": args.launch,
                    "iters": iters, "kmeans_iters": args.kmeans_iters,
                    "layout": "vector-major (nn.Linear [out, in])",
-                   "l2": "inputs larger than L2 (405 MB per step, distinct layer every step)",
+                   "l2": l2_note,
                    "parallelism": f"dp{world} (layers sharded over ranks, no exchange)"},
         "roofline": roofline,
-        "gpu_launches": args.steps * 7 * 2,   # decompose + table set-up per matrix
+        "gpu_launches": args.steps * launches_per_step,
         "clocks": clk,
     }
     if refinement is not None:
@@ -339,7 +416,7 @@ def run_gpu(args) -> dict:
     if e2e is not None:
         result["e2e"] = e2e
     if rank == 0 and world == 1 and not args.skip_cpu:
-        result["cpu_baseline"] = oracle_baseline(synth.llama7b_layer(0), iters, budget_s=args.cpu_budget,
+        result["cpu_baseline"] = oracle_baseline(layer_fn(0), iters, budget_s=args.cpu_budget,
                                                  kmeans_iters=args.kmeans_iters)
     if dist:
         dist.destroy_process_group()
@@ -460,26 +537,29 @@ def measure_rht(kd, torch, layer, stream):
                                "achieved": round(gbs_big, 1), "frac": round(gbs_big / peak, 4)}}
 
 
-def measure_refinement(kd, torch, layer, outs, wss, iters, stream, base_ms):
-    """Average N = 4096 launch time with KM_PROBE refinement iterations, against the
-    closed-form launch time measured in the timed region."""
-    evs = []
-    for rep in range(3):
-        for s, w in layer:
-            if s.N != 4096:
-                continue
-            a = torch.cuda.Event(enable_timing=True)
-            b = torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=outs[(s.N, s.M)], stream=stream,
-                         kmeans_iters=KM_PROBE)
-            b.record(stream)
-            if rep > 0:
-                evs.append((a, b))
-    torch.cuda.synchronize()
-    ms = sum(a.elapsed_time(b) for a, b in evs) / len(evs)
-    return {"kmeans_iters": KM_PROBE, "kernel": "decompose_kernel<N=4096>", "launch_ms": round(ms, 3),
-            "overhead_vs_closed_form": round(ms / base_ms - 1.0, 4)}
+def measure_refinement(kd, torch, layer, outs, wss, iters, stream, ndom):
+    """Cost of KM_PROBE Lloyd iterations on the dominant length: per-matrix launches
+    of that length with and without the refinement, timed back to back."""
+    def timed(km):
+        evs = []
+        for rep in range(3):
+            for i, (s, w) in enumerate(layer):
+                if s.N != ndom:
+                    continue
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], out=outs[i], stream=stream,
+                             kmeans_iters=km)
+                b.record(stream)
+                if rep > 0:
+                    evs.append((a, b))
+        torch.cuda.synchronize()
+        return sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+    base = timed(0)
+    ms = timed(KM_PROBE)
+    return {"kmeans_iters": KM_PROBE, "kernel": f"decompose_kernel<N={ndom}>", "launch_ms": round(ms, 3),
+            "closed_form_launch_ms": round(base, 3), "overhead_vs_closed_form": round(ms / base - 1.0, 4)}
 
 
 def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
@@ -492,9 +572,9 @@ def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
     for s, w in layer:   # two device input buffers per shape
         slots.setdefault(w.shape, [torch.empty_like(w, device=stream.device) for _ in range(2)])
     dev_out = [kd.Decomposed(
-        codes_u=torch.empty_like(outs[(s.N, s.M)].codes_u), codes_v=torch.empty_like(outs[(s.N, s.M)].codes_v),
-        centres_u=torch.empty_like(outs[(s.N, s.M)].centres_u), centres_v=torch.empty_like(outs[(s.N, s.M)].centres_v),
-        coeffs=None, u=None, vhat=None, resid=None, trace=None) for s, _ in layer]
+        codes_u=torch.empty_like(o.codes_u), codes_v=torch.empty_like(o.codes_v),
+        centres_u=torch.empty_like(o.centres_u), centres_v=torch.empty_like(o.centres_v),
+        coeffs=None, u=None, vhat=None, resid=None, trace=None) for o in outs]
     host_out = [tuple(torch.empty(t.shape, dtype=t.dtype).pin_memory()
                       for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v)) for o in dev_out]
     h2d = sum(w.numel() * w.element_size() for _, w in host_in)
@@ -573,7 +653,8 @@ def run_reference(args) -> dict | None:
     if rank != 0:
         return None
     from paper_2609_11687_gb300 import synth
-    specs = synth.llama7b_layer(0)
+    n_layers, layer_fn, workload_desc = _workloads()[args.workload]
+    specs = layer_fn(0)
     budget = max(1.0, min(30.0, 120.0 / max(1, args.steps + args.warmup)))
     vals = []
     for i in range(args.warmup + args.steps):
@@ -587,8 +668,8 @@ def run_reference(args) -> dict | None:
         "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": layer_params / value * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": "llama2-7b decoder layer per step (202,375,168 params), each timed step a "
-                               "bounded sample of that layer on the host cores", "iters": args.iters,
+        "config": {"workload": workload_desc + "; each timed step a bounded sample of that layer on the host "
+                               "cores", "iters": args.iters,
                    "kmeans_iters": args.kmeans_iters},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": os.cpu_count(), "kind": "oracle",
                          "sample": vals[-1]["sample"]},
@@ -630,6 +711,11 @@ def main():
     ap.add_argument("--kmeans-iters", type=int, default=0,
                     help="Lloyd refinement iterations of the centres (Sec. 2.1); 0 = closed form")
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--launch", default="batch", choices=["batch", "single"],
+                    help="one kd_decompose_batch launch per vector length (default) or one launch per matrix")
+    ap.add_argument("--workload", default="llama7b",
+                    choices=["llama7b", "w256", "opt125m", "pythia6.9b", "mistral7b"],
+                    help="synthetic stand-in per step (default: one Llama-2-7B-shaped layer)")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=12.0)

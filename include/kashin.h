@@ -136,6 +136,39 @@ kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, i
                               float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
                               void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Several matrices of one vector length n in one launch (Algorithm 1 and the 2-bit
+ * coding, as kd_decompose): the vector pairs of all matrices share the persistent
+ * CTAs, so small matrices fill the GPU and the last wave of one matrix overlaps the
+ * next.  Each matrix keeps its own sign seed, leading dimension and outputs; the
+ * arithmetic per vector pair is identical to kd_decompose's (bitwise equal results).
+ * Lengths n <= 8192 run as one launch; longer vectors (which fill the GPU alone)
+ * run one launch per matrix, in order, on the same stream and workspace.
+ *
+ *   mats      HOST array of `count` descriptors (1 <= count <= KD_MAX_BATCH); read
+ *             during the call only.  In each: w, m, ld, sign_seed as kd_decompose's
+ *             arguments; codes_u, codes_v, centres_u, centres_v required (m > 0);
+ *             coeffs optional (NULL).  No u / vhat / resid / trace outputs.
+ *   dtype, layout, n, iters, kmeans_iters   shared by all matrices.
+ *   workspace at least kd_workspace_size_batch(n, count) bytes.
+ * Errors as kd_decompose. */
+#define KD_MAX_BATCH 32
+typedef struct kd_matrix {
+  const void* w;
+  int64_t m;
+  int64_t ld;
+  uint64_t sign_seed;
+  uint32_t* codes_u;
+  uint32_t* codes_v;
+  float* centres_u;
+  float* centres_v;
+  float* coeffs;
+} kd_matrix;
+
+size_t kd_workspace_size_batch(int64_t n, int count);
+kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, kd_layout layout, int64_t n,
+                             int iters, int kmeans_iters, void* workspace, size_t ws_bytes, void* stream);
+
 /* y_j = P x_j for m vectors of length n, fp32, vector-major [m][n] contiguous
  * (Sec. 3.1: P z = IDCT(eps * DCT(z)); App. C uses the same operator on the rows
  * of the activations, XP).  x and y may alias. */

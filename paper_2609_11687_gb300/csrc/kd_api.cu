@@ -40,10 +40,31 @@ namespace {
 constexpr size_t kAlign = 256;
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
-// Workspace layout: [status word | pad][sign bits][access-ordered twiddles][u slots]
+// Workspace layout: [status word | pad][sign bits, one set per matrix][access-ordered twiddles][u slots]
 struct WsLayout {
   size_t status, eps, tw, uslots, total;
 };
+
+// sign bits of several matrices: set i at eps + i * words (batched launches)
+struct SeedList {
+  int count, words;
+  int64_t n;
+  uint64_t seed[kMaxBatch];
+};
+
+__global__ void eps_batch_kernel(uint32_t* eps, SeedList sl) {
+  const int total = sl.count * sl.words;
+  for (int g = blockIdx.x * blockDim.x + threadIdx.x; g < total; g += gridDim.x * blockDim.x) {
+    const int i = g / sl.words, wd = g - i * sl.words;
+    uint32_t bits = 0;
+    for (int bb = 0; bb < 32; ++bb) {
+      const int64_t j = (int64_t)wd * 32 + bb;
+      if (j >= sl.n) break;
+      bits |= (uint32_t)(splitmix64_mix(sl.seed[i] + (uint64_t)(j + 1) * 0x9E3779B97F4A7C15ull) >> 63) << bb;
+    }
+    eps[g] = bits;
+  }
+}
 
 int sm_count() {
   int dev = 0, sms = 0;
@@ -60,11 +81,11 @@ int max_decompose_ctas(const PlanOps* ops) {
   return per * sms;
 }
 
-bool layout_of(const PlanOps* ops, WsLayout* L) {
+bool layout_of(const PlanOps* ops, WsLayout* L, int nsets = 1) {
   const size_t n = (size_t)ops->n;
   L->status = 0;
   L->eps = kAlign;
-  L->tw = L->eps + align_up(((n + 31) / 32) * sizeof(uint32_t));
+  L->tw = L->eps + align_up((size_t)nsets * ((n + 31) / 32) * sizeof(uint32_t));
   L->uslots = L->tw + align_up((size_t)ops->twn * sizeof(float2));
   size_t us = 0;
   if (ops->u_in_gmem) {
@@ -178,7 +199,92 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
   const int ctas = max_decompose_ctas(ops);
   if (ctas <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, ctas);
-  return ops->decompose(p, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+  return ops->decompose(p, nullptr, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+size_t kd_workspace_size_batch(int64_t n, int count) {
+  const PlanOps* ops = plan_ops(n);
+  if (!ops || count < 1 || count > KD_MAX_BATCH) return 0;
+  WsLayout L;
+  if (!layout_of(ops, &L, count)) return 0;
+  return L.total;
+}
+
+kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, kd_layout layout, int64_t n,
+                             int iters, int kmeans_iters, void* workspace, size_t ws_bytes, void* stream) {
+  static_assert(KD_MAX_BATCH == kMaxBatch, "batch limit of the header and the kernel");
+  if (!mats || count < 1 || count > KD_MAX_BATCH || n <= 0 || iters < 0 || kmeans_iters < 0 ||
+      kmeans_iters > 64 || !valid_dtype(dtype) || !valid_layout(layout))
+    return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  BatchParams bp;
+  bp.count = count;
+  int64_t npairs = 0;
+  for (int i = 0; i < count; ++i) {
+    const kd_matrix& a = mats[i];
+    if (a.m < 0 || (layout == KD_VEC_ROWS ? a.ld < n : a.ld < a.m)) return KD_ERR_INVALID_ARG;
+    if (a.m > 0 && (!a.w || !a.codes_u || !a.codes_v || !a.centres_u || !a.centres_v)) return KD_ERR_INVALID_ARG;
+    BatchMat& b = bp.mat[i];
+    b.w = a.w;
+    b.m = a.m;
+    b.ld = a.ld;
+    b.pair0 = npairs;
+    b.codes_u = a.codes_u;
+    b.codes_v = a.codes_v;
+    b.centres_u = a.centres_u;
+    b.centres_v = a.centres_v;
+    b.coeffs = a.coeffs;
+    npairs += (a.m + 1) / 2;
+  }
+  WsLayout L;
+  if (!layout_of(ops, &L, count)) return KD_ERR_CUDA;
+  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!ops->batch) {
+    // long vectors: one launch per matrix on the same workspace, in stream order
+    for (int i = 0; i < count; ++i) {
+      const kd_matrix& a = mats[i];
+      const kd_status sti = kd_decompose(a.w, dtype, layout, n, a.m, a.ld, a.sign_seed, iters, kmeans_iters,
+                                         a.codes_u, a.codes_v, a.centres_u, a.centres_v, a.coeffs, nullptr,
+                                         nullptr, nullptr, nullptr, workspace, ws_bytes, stream);
+      if (sti != KD_OK) return sti;
+    }
+    return KD_OK;
+  }
+  kd_status st = setup(ops, L, workspace, mats[0].sign_seed, s);  // twiddles, status, set 0
+  if (st != KD_OK) return st;
+  char* b = static_cast<char*>(workspace);
+  SeedList sl;
+  sl.count = count;
+  sl.words = (int)((n + 31) / 32);
+  sl.n = n;
+  for (int i = 0; i < count; ++i) sl.seed[i] = mats[i].sign_seed;
+  if (count > 1) {  // set 0 came with the twiddles
+    const int total = count * sl.words;
+    eps_batch_kernel<<<(total + 255) / 256, 256, 0, s>>>(reinterpret_cast<uint32_t*>(b + L.eps), sl);
+    if (cudaGetLastError() != cudaSuccess) return KD_ERR_CUDA;
+  }
+  if (npairs == 0) return KD_OK;
+  DecParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.w = mats[0].w;
+  p.dtype = (int)dtype;
+  p.layout = (int)layout;
+  p.n = n;
+  p.m = mats[0].m;
+  p.ld = mats[0].ld;
+  p.iters = iters;
+  p.kmeans_iters = kmeans_iters;
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.status = reinterpret_cast<uint32_t*>(b + L.status);
+  p.uslots = ops->u_in_gmem ? reinterpret_cast<float2*>(b + L.uslots) : nullptr;
+  p.npairs = npairs;
+  const int ctas = max_decompose_ctas(ops);
+  if (ctas <= 0) return KD_ERR_CUDA;
+  const int grid = grid_for(p.npairs, ops->q, ctas);
+  return ops->decompose(p, &bp, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
 kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t sign_seed, void* workspace,

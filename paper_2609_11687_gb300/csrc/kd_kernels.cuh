@@ -187,6 +187,24 @@ struct DecParams {
   int64_t npairs;
 };
 
+// Several matrices of one vector length in one launch (kd_decompose_batch): their
+// pairs are numbered one after another; matrix i owns global pairs
+// [pair0, pair0 + ceil(m / 2)) and the sign bits at eps + i * ceil(n / 32).
+constexpr int kMaxBatch = 32;
+struct BatchMat {
+  const void* w;
+  int64_t m, ld, pair0;
+  uint32_t* codes_u;
+  uint32_t* codes_v;
+  float* centres_u;
+  float* centres_v;
+  float* coeffs;
+};
+struct BatchParams {
+  int count;  // 0: the single matrix of DecParams
+  BatchMat mat[kMaxBatch];
+};
+
 // sign(r) * c with sign(0) = 0
 __device__ __forceinline__ float signed_step(float r, float c) {
   return (r == 0.f) ? 0.f : copysignf(c, r);
@@ -196,7 +214,7 @@ __device__ __forceinline__ float signed_step(float r, float c) {
 // kd_decompose kernel
 // ---------------------------------------------------------------------------
 template <class PL, bool TRACE>
-__global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecParams p) {
+__global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecParams p, const __grid_constant__ BatchParams bp) {
   constexpr int N = PL::N;
   constexpr int T = PL::T;
   constexpr int E = PL::E;
@@ -217,12 +235,28 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
   if constexpr (PL::UMODE == UGMEM) uslot = p.uslots + ((int64_t)blockIdx.x * PL::Q + team) * N;
   if constexpr (PL::UMODE == USMEM) uslot = red + PL::RED;
 
+  int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
     const bool active = pair < p.npairs;
-    const int64_t pr = active ? pair : base;
+    int64_t pr = active ? pair : base;
+    // this pair's matrix: index mi into bp (batched launch) or DecParams' matrix;
+    // its fields are re-read from the parameter space where used (no registers held)
+    int mi = 0;
+    if (PL::BATCH && bp.count > 0) {
+      while (mi + 1 < bp.count && pr >= bp.mat[mi + 1].pair0) ++mi;
+      pr -= bp.mat[mi].pair0;
+      if (mi != cur_mat) {  // uniform per team: Q == 1 whenever T > 32
+        xf.set_eps(p.eps + (int64_t)mi * ((N + 31) / 32));
+        cur_mat = mi;
+      }
+    }
+    const bool batched = PL::BATCH && bp.count > 0;
+    auto w_in = [&]() -> const void* { return batched ? bp.mat[mi].w : p.w; };
+    auto ld_in = [&]() -> int64_t { return batched ? bp.mat[mi].ld : p.ld; };
+    const int64_t m_in = batched ? bp.mat[mi].m : p.m;
     const int64_t colA = 2 * pr;
-    const bool hasB = (colA + 1) < p.m;
+    const bool hasB = (colA + 1) < m_in;
     const int64_t colB = hasB ? colA + 1 : colA;
 
     // ---- load the pair in Makhoul order: position lt + j*T ----
@@ -231,8 +265,8 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
-      const float a = load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld));
-      const float b = hasB ? load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)) : 0.f;
+      const float a = load_elem(w_in(), p.dtype, elem_index(p.layout, colA, nat, ld_in()));
+      const float b = hasB ? load_elem(w_in(), p.dtype, elem_index(p.layout, colB, nat, ld_in())) : 0.f;
       r[j] = make_float2(a, b);
       acc.x = __fadd_rn(acc.x, fabsf(a));
       acc.y = __fadd_rn(acc.y, fabsf(b));
@@ -347,9 +381,9 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
 #pragma unroll
         for (int j = 0; j < E; ++j) {
           const int nat = nat_of<N>(lt + j * T);
-          const float a = __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colA, nat, p.ld)), scA);
+          const float a = __fmul_rn(load_elem(w_in(), p.dtype, elem_index(p.layout, colA, nat, ld_in())), scA);
           const float b =
-              hasB ? __fmul_rn(load_elem(p.w, p.dtype, elem_index(p.layout, colB, nat, p.ld)), scB) : 0.f;
+              hasB ? __fmul_rn(load_elem(w_in(), p.dtype, elem_index(p.layout, colB, nat, ld_in())), scB) : 0.f;
           const float2 uj = u_at(j);
           r[j] = make_float2(__fsub_rn(__fsub_rn(a, uj.x), r[j].x), __fsub_rn(__fsub_rn(b, uj.y), r[j].y));
         }
@@ -541,7 +575,8 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         const bool isB = (plane & 1) != 0;
         if (isB && !hasB) continue;
         const int64_t col = isB ? colB : colA;
-        uint32_t* dst = (plane < 2) ? p.codes_u : p.codes_v;
+        uint32_t* dst = (plane < 2) ? (batched ? bp.mat[mi].codes_u : p.codes_u)
+                                    : (batched ? bp.mat[mi].codes_v : p.codes_v);
         dst[col * WPV + word] = packed;
       }
       if (lt == 0) {
@@ -551,15 +586,16 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
           const float c1 = v2 ? coef[0].y : coef[0].x, c2 = v2 ? coef[1].y : coef[1].x;
           const float d1 = v2 ? coef[2].y : coef[2].x, d2 = v2 ? coef[3].y : coef[3].x;
           const float f = sc[v2];
-          float* cu = p.centres_u + col * 4;
-          float* cv = p.centres_v + col * 4;
+          float* cu = (batched ? bp.mat[mi].centres_u : p.centres_u) + col * 4;
+          float* cv = (batched ? bp.mat[mi].centres_v : p.centres_v) + col * 4;
+          float* coeffs_out = batched ? bp.mat[mi].coeffs : p.coeffs;
 #pragma unroll
           for (int qq = 0; qq < 4; ++qq) {
             cu[qq] = __fmul_rn(cen[0][v2][qq], f);
             cv[qq] = __fmul_rn(cen[1][v2][qq], f);
           }
-          if (p.coeffs) {
-            float* co = p.coeffs + col * 4;
+          if (coeffs_out) {
+            float* co = coeffs_out + col * 4;
             co[0] = __fmul_rn(c1, f); co[1] = __fmul_rn(c2, f);
             co[2] = __fmul_rn(d1, f); co[3] = __fmul_rn(d2, f);
           }

@@ -24,11 +24,16 @@ inline int occupancy(K kernel, int threads, size_t smem) {
 
 template <class PL>
 struct Ops {
-  static cudaError_t decompose(const DecParams& p, int grid, cudaStream_t s) {
+  static cudaError_t decompose(const DecParams& p, const BatchParams* bp, int grid, cudaStream_t s) {
     auto k = p.trace ? decompose_kernel<PL, true> : decompose_kernel<PL, false>;
     cudaError_t e = prepare(k, PL::SMEM);
     if (e != cudaSuccess) return e;
-    k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
+    if (bp) {
+      k<<<grid, PL::THREADS, PL::SMEM, s>>>(p, *bp);
+    } else {
+      BatchParams none{};
+      k<<<grid, PL::THREADS, PL::SMEM, s>>>(p, none);
+    }
     return cudaGetLastError();
   }
   static cudaError_t reconstruct(const RecParams& p, int grid, cudaStream_t s) {
@@ -58,7 +63,7 @@ struct Ops {
     return occupancy(reconstruct_kernel<PL>, PL::THREADS, PL::SMEM);
   }
   static const PlanOps* ops() {
-    static const PlanOps o{PL::N, PL::THREADS, PL::Q, PL::SMEM, PL::UMODE == UGMEM, PL::TWN,
+    static const PlanOps o{PL::N, PL::THREADS, PL::Q, PL::SMEM, PL::UMODE == UGMEM, PL::BATCH, PL::TWN,
                            &Ops::ctas_per_sm, &Ops::decompose, &Ops::apply, &Ops::reconstruct, &Ops::setup};
     return &o;
   }

@@ -7,6 +7,7 @@
 
 namespace kd {
 struct DecParams;
+struct BatchParams;
 struct ApplyParams;
 struct RecParams;
 
@@ -16,10 +17,12 @@ struct PlanOps {
   int q;            // vector pairs per CTA per iteration
   size_t smem;      // dynamic shared memory per CTA
   bool u_in_gmem;   // u lives in per-team workspace slots
+  bool batch;       // the decompose kernel takes several matrices per launch
   int twn;          // entries of the access-ordered twiddle table
   // CTAs that fit on one SM (occupancy), 0 on error
   int (*ctas_per_sm)(int which);  // which: 0 decompose, 1 apply, 2 reconstruct
-  cudaError_t (*decompose)(const DecParams&, int grid, cudaStream_t);
+  // bp: the matrices of a batched launch, or nullptr for DecParams' single matrix
+  cudaError_t (*decompose)(const DecParams&, const BatchParams* bp, int grid, cudaStream_t);
   cudaError_t (*apply)(const ApplyParams&, int grid, cudaStream_t);
   cudaError_t (*reconstruct)(const RecParams&, int grid, cudaStream_t);
   // tables for one call: twiddles (float2[twn]), sign bits, cleared status word

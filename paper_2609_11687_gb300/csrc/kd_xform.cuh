@@ -81,6 +81,9 @@ struct Plan {
   static constexpr int E = Rv[0];
   static constexpr int RL = Rv[NP - 1];
   static constexpr int THREADS = T * Q;
+  // batched launches (kd_decompose_batch) compiled in: the lengths whose matrices can
+  // be too small to fill the GPU alone (longer ones run one launch per matrix)
+  static constexpr bool BATCH = N_ <= 8192;
   static constexpr int NW = (T + 31) / 32;  // warps per team
   static constexpr int BUF = (N + N / 16 + N / 256 + 8 + 15) / 16 * 16;  // padded float2 slots per team
   // float2 reduction slots per team: ping-pong partials of team_sum, or the
@@ -229,7 +232,6 @@ struct Xform {
     tw = t;
     lt = lane_t;
     pb0 = pad(lt);
-    ek = em = 0;
     if constexpr (PL::PAIRED) {
       constexpr int H = PL::HALF;
       constexpr int L = T;
@@ -239,14 +241,7 @@ struct Xform {
       self = (bb == 0) ? (h == 0 ? 1 : 2) : 0;
       lbase = slot_low<PL>(kgrp);
       cw = expi_pi(kgrp, N);
-#pragma unroll
-      for (int kp = 0; kp < E; ++kp) {
-        const int k = kgrp + L * kp;
-        ek |= (Mask)eps_neg(eb, k) << kp;
-        em |= (Mask)eps_neg(eb, (N - k) % N) << kp;
-      }
       p0 = p1 = pbp0 = pbp1 = 0;
-      dm = ek ^ em;
     } else {
       const int Kp = rest_of_slot<PL>(lt);
       p0 = slot_rest<PL>((T - Kp) % T);
@@ -254,15 +249,31 @@ struct Xform {
       pbp0 = pad(p0);
       pbp1 = pad(p1);
       cw = expi_pi((long long)E * Kp, N);
+      kgrp = self = lbase = 0;
+    }
+    set_eps(eb);
+  }
+
+  // the sign set's bits at this thread's frequencies (and their mirrors)
+  __device__ __forceinline__ void set_eps(const uint32_t* __restrict__ eb) {
+    ek = em = 0;
+    if constexpr (PL::PAIRED) {
+#pragma unroll
+      for (int kp = 0; kp < E; ++kp) {
+        const int k = kgrp + T * kp;
+        ek |= (Mask)eps_neg(eb, k) << kp;
+        em |= (Mask)eps_neg(eb, (N - k) % N) << kp;
+      }
+    } else {
+      const int Kp = rest_of_slot<PL>(lt);
 #pragma unroll
       for (int r = 0; r < E; ++r) {
         const int k = r + E * Kp;
         ek |= (Mask)eps_neg(eb, k) << r;
         em |= (Mask)eps_neg(eb, (N - k) % N) << r;
       }
-      kgrp = self = lbase = 0;
-      dm = ek ^ em;
     }
+    dm = ek ^ em;
   }
 
   // padded address of pass-0 slot lt + j T (base + compile-time offset when separable)

@@ -31,7 +31,16 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
-           "kd_rht_block", "kd_rht", "kd_dequantise", "kd_measure_fp32_peak")
+           "kd_rht_block", "kd_rht", "kd_dequantise", "kd_measure_fp32_peak", "kd_workspace_size_batch",
+           "kd_decompose_batch")
+KD_MAX_BATCH = 32
+
+
+class KdMatrix(ctypes.Structure):
+    """Mirror of kd_matrix (include/kashin.h)."""
+    _fields_ = [("w", ctypes.c_void_p), ("m", ctypes.c_int64), ("ld", ctypes.c_int64),
+                ("sign_seed", ctypes.c_uint64), ("codes_u", ctypes.c_void_p), ("codes_v", ctypes.c_void_p),
+                ("centres_u", ctypes.c_void_p), ("centres_v", ctypes.c_void_p), ("coeffs", ctypes.c_void_p)]
 
 
 def _load() -> ctypes.CDLL:
@@ -60,6 +69,10 @@ def _load() -> ctypes.CDLL:
     lib.kd_reconstruct.restype = c_int
     lib.kd_read_status.argtypes = [c_vp, c_vp]
     lib.kd_read_status.restype = c_int
+    lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
+    lib.kd_workspace_size_batch.restype = c_sz
+    lib.kd_decompose_batch.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
+    lib.kd_decompose_batch.restype = c_int
     lib.kd_measure_fp32_peak.argtypes = [c_vp, c_vp]
     lib.kd_measure_fp32_peak.restype = c_int
     lib.kd_dequantise.argtypes = [c_vp, c_vp, c_i64, c_i64, c_int, c_int, c_vp, c_i64, c_vp]
@@ -127,6 +140,20 @@ def kd_reconstruct(codes_u, codes_v, centres_u, centres_v, n, m, sign_seed, out_
                               workspace, ws_bytes, stream)
 
 
+def kd_batchable(n: int) -> bool:
+    """True when kd_decompose_batch runs all matrices of length n in one launch
+    (n <= 8192, as include/kashin.h states); longer vectors run one launch each."""
+    return kd_supported(n) == KD_OK and int(n) <= 8192
+
+
+def kd_workspace_size_batch(n: int, count: int) -> int:
+    return int(lib.kd_workspace_size_batch(int(n), int(count)))
+
+
+def kd_decompose_batch(mats, count, dtype, layout, n, iters, kmeans_iters, workspace, ws_bytes, stream) -> int:
+    return lib.kd_decompose_batch(mats, count, dtype, layout, n, iters, kmeans_iters, workspace, ws_bytes, stream)
+
+
 def kd_read_status(workspace, stream) -> int:
     return lib.kd_read_status(workspace, stream)
 
@@ -183,10 +210,11 @@ def _stream(stream) -> int:
 class Workspace:
     """Device scratch for one vector length (reusable across calls on one stream)."""
 
-    def __init__(self, n: int, device="cuda"):
+    def __init__(self, n: int, device="cuda", count: int = 1):
         torch = _torch()
         self.n = int(n)
-        size = kd_workspace_size(self.n)
+        self.count = int(count)
+        size = kd_workspace_size(self.n) if self.count == 1 else kd_workspace_size_batch(self.n, self.count)
         if size == 0:
             raise KashinError(KD_ERR_UNSUPPORTED_N if kd_supported(self.n) else KD_ERR_CUDA,
                               f"kd_workspace_size({self.n})")
@@ -252,6 +280,46 @@ def decompose(w, iters: int, sign_seed: int, layout: str = "rows", factors: bool
     if st != KD_OK:
         raise KashinError(st, "kd_decompose")
     return out
+
+
+def decompose_batch(ws, iters: int, sign_seeds, layout: str = "rows", coeffs: bool = False,
+                    workspace: Optional[Workspace] = None, outs=None, stream=None, kmeans_iters: int = 0):
+    """Decompose and code several matrices of one vector length in one launch
+    (kd_decompose_batch): ``ws`` is a list of up to KD_MAX_BATCH CUDA tensors of one
+    dtype and layout, ``sign_seeds`` their seeds.  Returns one Decomposed per matrix
+    (no factor or trace outputs)."""
+    torch = _torch()
+    if not 1 <= len(ws) <= KD_MAX_BATCH or len(sign_seeds) != len(ws):
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices with one seed each")
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    n = ws[0].shape[1] if lay == KD_VEC_ROWS else ws[0].shape[0]
+    dt = ws[0].dtype
+    arr = (KdMatrix * len(ws))()
+    res = []
+    for i, w in enumerate(ws):
+        if not w.is_cuda or w.dim() != 2 or w.stride(1) != 1 or w.dtype != dt:
+            raise ValueError("matrices must be 2-D CUDA tensors of one dtype with unit inner stride")
+        m = w.shape[0] if lay == KD_VEC_ROWS else w.shape[1]
+        if (w.shape[1] if lay == KD_VEC_ROWS else w.shape[0]) != n:
+            raise ValueError("matrices must share the vector length")
+        if outs is not None:
+            o = outs[i]
+        else:
+            f32 = dict(dtype=torch.float32, device=w.device)
+            o = Decomposed(codes_u=torch.empty((m, (n + 15) // 16), dtype=torch.int32, device=w.device),
+                           codes_v=torch.empty((m, (n + 15) // 16), dtype=torch.int32, device=w.device),
+                           centres_u=torch.empty((m, 4), **f32), centres_v=torch.empty((m, 4), **f32),
+                           coeffs=torch.empty((m, 4), **f32) if coeffs else None,
+                           u=None, vhat=None, resid=None, trace=None)
+        arr[i] = KdMatrix(w.data_ptr(), m, w.stride(0), int(sign_seeds[i]) & ((1 << 64) - 1),
+                          _ptr(o.codes_u), _ptr(o.codes_v), _ptr(o.centres_u), _ptr(o.centres_v), _ptr(o.coeffs))
+        res.append(o)
+    wsp = workspace if workspace is not None else Workspace(n, ws[0].device, count=len(ws))
+    st = kd_decompose_batch(ctypes.cast(arr, ctypes.c_void_p), len(ws), _dtype_code(dt), lay, n, int(iters),
+                            int(kmeans_iters), wsp.ptr, wsp.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_decompose_batch")
+    return res
 
 
 def read_status(workspace: Workspace, stream=None) -> int:

@@ -121,6 +121,31 @@ def test_rht_block_and_validation(kd):
     assert kd.kd_rht(null, 0, 256, 0, 256, 0, 0, null, 256, null, null) == kd.KD_OK
 
 
+def test_batch_workspace_and_validation(kd):
+    import ctypes
+    for n in (256, 768, 4096):
+        one = kd.kd_workspace_size(n)
+        assert kd.kd_workspace_size_batch(n, 1) == one
+        big = kd.kd_workspace_size_batch(n, 32)
+        assert big > one and big >= 256 + 32 * (n // 8) + 8 * n   # status, 32 sign sets, twiddles
+    assert kd.kd_workspace_size_batch(4096, 0) == 0 and kd.kd_workspace_size_batch(4096, 33) == 0
+    assert kd.kd_workspace_size_batch(100, 2) == 0
+    arr = (kd.KdMatrix * 2)()
+    for i in range(2):
+        arr[i] = kd.KdMatrix(None, 0, 4096, i, None, None, None, None, None)
+    ptr = ctypes.cast(arr, ctypes.c_void_p)
+    null = None
+    assert kd.kd_decompose_batch(ptr, 0, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose_batch(ptr, 33, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose_batch(null, 2, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4095, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_UNSUPPORTED_N
+    assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4096, 4, 0, 1, 16, null) == kd.KD_ERR_WORKSPACE
+    arr[1] = kd.KdMatrix(None, 3, 4096, 1, None, None, None, None, None)   # m > 0 without pointers
+    assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
+    arr[1] = kd.KdMatrix(1, 3, 4095, 1, 1, 1, 1, 1, None)                  # ld < n
+    assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
+
+
 def test_dequantise_validation(kd):
     null = None
     assert kd.kd_dequantise(16, 16, 0, 4, 0, 0, 16, 16, null) == kd.KD_ERR_INVALID_ARG
