@@ -91,11 +91,7 @@ struct Plan {
   static constexpr int RED = (4 * NW > 8 * (NW + 1)) ? 4 * NW : 8 * (NW + 1);
   static constexpr int USL = (UMODE_ == 2) ? N : 0;            // float2 slots of u per team (shared)
   // M in registers: one last-pass group per thread, partner at lane ^ HALF
-#ifdef KD_NO_PAIRED
-  static constexpr bool PAIRED = false;
-#else
   static constexpr bool PAIRED = (RL == E) && (N / RL == T);
-#endif
   static constexpr int HALF = (T < 32 ? T : 32) / 2;
 
   KD_HD static constexpr int R(int i) { return Rv[i]; }
