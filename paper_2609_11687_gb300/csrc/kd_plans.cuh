@@ -14,7 +14,7 @@ using Plan64 = Plan<64, 8, 4, UREG, 8, 8, 8>;
 using Plan128 = Plan<128, 8, 4, UREG, 8, 16, 8>;
 using Plan256 = Plan<256, 16, 4, USMEM, 8, 16, 16>;
 using Plan512 = Plan<512, 32, 2, USMEM, 8, 16, 32>;
-using Plan768 = Plan<768, 32, 2, USMEM, 4, 24, 32>;
+using Plan768 = Plan<768, 32, 2, USMEM, 6, 24, 32>;
 using Plan1024 = Plan<1024, 64, 1, USMEM, 8, 16, 8, 8>;
 using Plan1536 = Plan<1536, 96, 1, USMEM, 5, 16, 12, 8>;
 using Plan2048 = Plan<2048, 128, 1, USMEM, 4, 16, 16, 8>;
