@@ -565,12 +565,18 @@ def measure_refinement(kd, torch, layer, outs, wss, iters, stream, ndom):
 def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
     """Same metric through the C ABI with host buffers: every step copies the
     layer's fp16 weights from pinned host memory and reads codes + centres back.
-    Copies run on their own streams, double-buffered, so matrix i + 1 uploads and
-    matrix i - 1 downloads while matrix i decomposes."""
+    The matrices of one vector length form a group that goes out as one
+    kd_decompose_batch (as in the timed region); uploads, decompositions and
+    downloads run on three streams with two device copies of every group's inputs,
+    so one group uploads while another decomposes."""
     host_in = [(s, w.cpu().pin_memory()) for s, w in layer]
-    slots = {}
-    for s, w in layer:   # two device input buffers per shape
-        slots.setdefault(w.shape, [torch.empty_like(w, device=stream.device) for _ in range(2)])
+    groups = {}
+    for i, (s, _) in enumerate(layer):
+        groups.setdefault(s.N, []).append(i)
+    gorder = list(groups)
+    wsb = {n_: kd.Workspace(n_, stream.device, count=len(ix)) for n_, ix in groups.items()}
+    slots = {n_: [[torch.empty_like(host_in[i][1], device=stream.device) for i in ix] for _ in range(2)]
+             for n_, ix in groups.items()}
     dev_out = [kd.Decomposed(
         codes_u=torch.empty_like(o.codes_u), codes_v=torch.empty_like(o.codes_v),
         centres_u=torch.empty_like(o.centres_u), centres_v=torch.empty_like(o.centres_v),
@@ -581,38 +587,39 @@ def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
     d2h = sum(t.numel() * t.element_size() for o in dev_out for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v))
     up = torch.cuda.Stream(device=stream.device)
     down = torch.cuda.Stream(device=stream.device)
-    # freed[shape][slot]: the decompose that last read that slot has finished
-    freed = {k: [None, None] for k in slots}
-    use = {k: 0 for k in slots}
-    # read[i]: matrix i's outputs have been copied to the host (they may be rewritten)
-    read = [None] * len(layer)
+    freed = {n_: [None, None] for n_ in groups}   # the launch that last read that input copy is done
+    use = {n_: 0 for n_ in groups}
+    read = {n_: None for n_ in groups}            # the group's outputs reached the host
 
     def step():
-        for j, ((s, hw), o, ho) in enumerate(zip(host_in, dev_out, host_out)):
-            k = hw.shape
-            i = use[k] % 2
-            use[k] += 1
-            dw = slots[k][i]
+        for n_ in gorder:
+            ix = groups[n_]
+            k = use[n_] % 2
+            use[n_] += 1
+            dws = slots[n_][k]
             with torch.cuda.stream(up):
-                if freed[k][i] is not None:
-                    up.wait_event(freed[k][i])
-                dw.copy_(hw, non_blocking=True)
+                if freed[n_][k] is not None:
+                    up.wait_event(freed[n_][k])
+                for i, dw in zip(ix, dws):
+                    dw.copy_(host_in[i][1], non_blocking=True)
                 loaded = torch.cuda.Event()
                 loaded.record(up)
             stream.wait_event(loaded)
-            if read[j] is not None:
-                stream.wait_event(read[j])
-            kd.decompose(dw, iters, s.sign_seed, workspace=wss[s.N], out=o, stream=stream,
-                         kmeans_iters=args.kmeans_iters)
+            if read[n_] is not None:
+                stream.wait_event(read[n_])
+            kd.decompose_batch(dws, iters, [host_in[i][0].sign_seed for i in ix], workspace=wsb[n_],
+                               outs=[dev_out[i] for i in ix], stream=stream, kmeans_iters=args.kmeans_iters)
             done = torch.cuda.Event()
             done.record(stream)
-            freed[k][i] = done
+            freed[n_][k] = done
             with torch.cuda.stream(down):
                 down.wait_event(done)
-                for h, t in zip(ho, (o.codes_u, o.codes_v, o.centres_u, o.centres_v)):
-                    h.copy_(t, non_blocking=True)
-                read[j] = torch.cuda.Event()
-                read[j].record(down)
+                for i in ix:
+                    o = dev_out[i]
+                    for h, t in zip(host_out[i], (o.codes_u, o.codes_v, o.centres_u, o.centres_v)):
+                        h.copy_(t, non_blocking=True)
+                read[n_] = torch.cuda.Event()
+                read[n_].record(down)
 
     def drain():
         fin = torch.cuda.Event()
@@ -641,7 +648,8 @@ def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
     ms, total = shard.aggregate(a.elapsed_time(b), n * params)
     return {"value": round(total / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": n,
-            "pipeline": "H2D, decompose and D2H on three streams, double-buffered inputs"}
+            "pipeline": "per vector length: H2D, one batched decompose and D2H on three streams, two copies of "
+                        "the inputs"}
 
 
 # ---------------------------------------------------------------------------
