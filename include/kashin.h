@@ -88,8 +88,8 @@ kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host);
  *  iters      k >= 0 blocks of four atomic greedy steps (two on Q_N -> u, two on
  *             P Q_N -> vhat).  k = 0 gives zero factors, zero centres, codes 0.
  *  kmeans_iters  0..64 Lloyd refinement iterations of each factor's 4 centres from
- *             the closed form (Sec. 2.1: "a small number of k-means refinement
- *             iterations"): every entry goes to its nearest centre (ties to the
+ *             the closed form (Sec. 2.1 refines the closed-form centres with a few
+ *             k-means iterations): every entry goes to its nearest centre (ties to the
  *             lower), each centre becomes its cluster's mean, an empty cluster keeps
  *             its centre.  0 = the closed-form centres alone.
  *  codes_u,   required, uint32[m][ceil(n/16)]: 2-bit code of u_i (resp. vhat_i) at

@@ -12,8 +12,8 @@ Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
                               App. C footnote).  Row 0 carries the extra ``1/sqrt 2``
                               that makes the matrix orthogonal (the printed formula omits it).
 * ``sign_mask``            -- the per-matrix sign set ``epsilon`` (Sec. 3.1 ``T_E``;
-                              App. C "generated once from a fixed seed").  The paper
-                              does not name its generator; this build reads it as
+                              App. C: drawn once per layer from a fixed seed).  The paper
+                              does not name its generator; the oracle takes it to be
                               SplitMix64 (Steele, Lea & Flood, OOPSLA 2014): bit 63 of
                               the mix of ``seed + (j + 1) * gamma`` set means -1.
 * ``apply_p``              -- ``P z = IDCT(eps * DCT(z))`` with the dense matrix (Alg. 1).
@@ -22,9 +22,9 @@ Everything is float64 NumPy with an explicit ``N x N`` DCT-II matrix:
                               step divisor ``N`` as printed.  Optional tie-follow.
 * ``centres`` / ``codes``  -- the closed-form centres +-c1 +-c2 (Sec. 2.1) and the
                               nearest-centre 2-bit code (Sec. 2.1, App. C).
-* ``kmeans_refine``        -- the "small number of k-means refinement iterations" that
-                              Sec. 2.1 runs from the closed-form centres: 1-D Lloyd steps
-                              with 4 centres, an empty cluster keeps its centre.
+* ``kmeans_refine``        -- the few k-means refinement iterations that Sec. 2.1 runs
+                              from the closed-form centres: 1-D Lloyd steps with 4
+                              centres, an empty cluster keeps its centre.
 * ``reconstruct``          -- dequantised ``W_hat = U_q + P V_q`` (App. C, Eq. 11).
 * ``randomized_hadamard``  -- the randomized-Hadamard incoherence rotation that the
                               Kashin-DCT+H pipeline applies to a weight matrix before the
