@@ -101,9 +101,10 @@ def test_iteration_counts(kd, torch_mod, iters):
         assert not dev["words_u"].any() and not dev["words_v"].any()
 
 
-@pytest.mark.parametrize("n,m", [(16, 3), (64, 5), (768, 13), (3072, 9), (4096, 13), (11008, 5), (14336, 3),
-                                 (16384, 3)])
+@pytest.mark.parametrize("n,m", [(16, 3), (32, 7), (64, 5), (128, 5), (768, 13), (1024, 3), (1536, 5), (2048, 3),
+                                 (3072, 9), (4096, 13), (8192, 3), (11008, 5), (14336, 3), (16384, 3)])
 def test_shapes_ragged(kd, torch_mod, n, m):
+    """Every compiled plan against the oracle, odd vector counts (a lone last vector)."""
     torch = torch_mod
     G = _rand(torch, (m, n), seed=n + m)
     rep, _ = _parity(kd, torch, G, seed=n)
