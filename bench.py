@@ -686,14 +686,16 @@ def run_reference(args) -> dict | None:
 
 
 def run_profile_case(args) -> None:
-    """Small case for ncu: one matrix of the layer's distribution with M vectors
-    (default q: n = 4096, M = 32768, 256 MB of input, above L2), decomposed 3 times."""
+    """Small case for ncu: one matrix of the workload's layer with M vectors (default
+    the 7B layer's q: n = 4096, M = 32768, 256 MB of input, above L2), decomposed 3
+    times."""
     import dataclasses
     import torch
     from paper_2609_11687_gb300 import build, synth
     build.build()
     from paper_2609_11687_gb300 import kashin as kd
-    spec = dataclasses.replace(synth.llama7b_layer(0)[args.profile_matrix], M=args.profile_m)
+    layer_fn = _workloads()[args.workload][1]
+    spec = dataclasses.replace(layer_fn(0)[args.profile_matrix], M=args.profile_m)
     w = synth.generate(spec, device="cuda")
     if args.profile_kernel == "rht":
         y = torch.empty(w.shape, dtype=torch.float32, device="cuda")
