@@ -394,14 +394,23 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         }
         team_sync<PL>();  // the last transform's readers of buf are done
       } else if ((hb & 1) == 0) {
-        // two greedy steps from Q_N (update u).  With u outside registers, step 1's
-        // signs are kept as bits and u is updated once after step 2 as
-        // (u + d1) + d2 -- the same roundings as two separate updates.
+        // two greedy steps from Q_N (update u)
         Bits nzA = 0, ngA = 0, nzB = 0, ngB = 0;
         float2 l1 = make_float2(0.f, 0.f);
+        // u in shared memory: both steps update it in place (two roundings, as
+        // with two separate updates); u in the workspace: step 1 keeps its signs
+        // as bits and step 2 applies (u + d1) + d2 in one read-modify-write
+        auto add_smem = [&](int j, float dA, float dB) {
+          float2 uj = uslot[lt + j * T];
+          uj.x = __fadd_rn(uj.x, dA);
+          uj.y = __fadd_rn(uj.y, dB);
+          uslot[lt + j * T] = uj;
+        };
         auto rec1 = [&](int j, float dA, float dB) {
           if constexpr (PL::UMODE == UREG) {
             add_u(j, dA, dB);
+          } else if constexpr (PL::UMODE == USMEM) {
+            add_smem(j, dA, dB);
           } else {
             nzA |= (Bits)(dA != 0.f) << j;
             ngA |= (Bits)(__float_as_uint(dA) >> 31) << j;
@@ -412,6 +421,8 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         auto upd2 = [&](int j, float dA, float dB) {
           if constexpr (PL::UMODE == UREG) {
             add_u(j, dA, dB);
+          } else if constexpr (PL::UMODE == USMEM) {
+            add_smem(j, dA, dB);
           } else {
             const float d1A = ((nzA >> j) & 1u) ? __uint_as_float(__float_as_uint(l1.x) | (uint32_t)((ngA >> j) & 1u) << 31) : 0.f;
             const float d1B = ((nzB >> j) & 1u) ? __uint_as_float(__float_as_uint(l1.y) | (uint32_t)((ngB >> j) & 1u) << 31) : 0.f;
