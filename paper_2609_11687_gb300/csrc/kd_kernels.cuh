@@ -365,7 +365,6 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
     // Half-block hb: even = two greedy steps from Q_N (u), odd = two from P Q_N (vhat),
     // each followed by P; the last one (hb == 2k) forms x - u - r and its P gives vhat.
     // One call site for the transform keeps the kernel's code footprint small.
-    using Bits = typename std::conditional<(E > 32), uint64_t, uint32_t>::type;
     int step = 0;
     const int HB = 2 * p.iters;
     for (int hb = 0; hb <= HB; ++hb) {
@@ -395,46 +394,23 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         team_sync<PL>();  // the last transform's readers of buf are done
       } else if ((hb & 1) == 0) {
         // two greedy steps from Q_N (update u)
-        Bits nzA = 0, ngA = 0, nzB = 0, ngB = 0;
         float2 l1 = make_float2(0.f, 0.f);
-        // u in shared memory: both steps update it in place (two roundings, as
-        // with two separate updates); u in the workspace: step 1 keeps its signs
-        // as bits and step 2 applies (u + d1) + d2 in one read-modify-write
-        auto add_smem = [&](int j, float dA, float dB) {
-          float2 uj = uslot[lt + j * T];
-          uj.x = __fadd_rn(uj.x, dA);
-          uj.y = __fadd_rn(uj.y, dB);
-          uslot[lt + j * T] = uj;
-        };
-        auto rec1 = [&](int j, float dA, float dB) {
+        // u outside registers (shared memory, or the workspace slot for the longest
+        // vectors) is updated in place by both steps: two roundings, as with two
+        // separate updates
+        auto add_slot = [&](int j, float dA, float dB) {
           if constexpr (PL::UMODE == UREG) {
             add_u(j, dA, dB);
-          } else if constexpr (PL::UMODE == USMEM) {
-            add_smem(j, dA, dB);
           } else {
-            nzA |= (Bits)(dA != 0.f) << j;
-            ngA |= (Bits)(__float_as_uint(dA) >> 31) << j;
-            nzB |= (Bits)(dB != 0.f) << j;
-            ngB |= (Bits)(__float_as_uint(dB) >> 31) << j;
-          }
-        };
-        auto upd2 = [&](int j, float dA, float dB) {
-          if constexpr (PL::UMODE == UREG) {
-            add_u(j, dA, dB);
-          } else if constexpr (PL::UMODE == USMEM) {
-            add_smem(j, dA, dB);
-          } else {
-            const float d1A = ((nzA >> j) & 1u) ? __uint_as_float(__float_as_uint(l1.x) | (uint32_t)((ngA >> j) & 1u) << 31) : 0.f;
-            const float d1B = ((nzB >> j) & 1u) ? __uint_as_float(__float_as_uint(l1.y) | (uint32_t)((ngB >> j) & 1u) << 31) : 0.f;
             float2 uj = uslot[lt + j * T];
-            uj.x = __fadd_rn(__fadd_rn(uj.x, d1A), dA);
-            uj.y = __fadd_rn(__fadd_rn(uj.y, d1B), dB);
+            uj.x = __fadd_rn(uj.x, dA);
+            uj.y = __fadd_rn(uj.y, dB);
             uslot[lt + j * T] = uj;
           }
         };
-        l1 = greedy(step, hb == 0, sum0, rec1);
+        l1 = greedy(step, hb == 0, sum0, add_slot);
         ++step;
-        const float2 l2 = greedy(step, false, sum0, upd2);
+        const float2 l2 = greedy(step, false, sum0, add_slot);
         ++step;
         if (hb == 0) {
           coef[0] = l1;
