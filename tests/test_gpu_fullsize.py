@@ -73,3 +73,29 @@ def test_fullsize_sampled_parity(kd, cfg, spec):
 @pytest.mark.parametrize("cfg,spec", KM_CASES, ids=[f"{c}-{s.name}" for c, s in KM_CASES])
 def test_fullsize_sampled_parity_kmeans(kd, cfg, spec):
     _run(kd, cfg, spec, kmeans_iters=3)
+
+
+def test_beyond_2_31_entries_int64_indexing(kd):
+    """A matrix of more than 2^31 entries (n = 4096, m = 524,291 vectors, 4.3 GB of
+    fp16): vectors at the far end, whose element offsets exceed 2^31, must come out
+    bitwise equal to a decomposition of just those vectors.  Empty inputs are legal."""
+    import torch
+    n, m = 4096, (1 << 19) + 3
+    assert n * m > 2**31
+    g = torch.Generator(device="cuda").manual_seed(11)
+    w = (torch.randn((m, n), generator=g, device="cuda", dtype=torch.float32) * 0.02).half()
+    full = kd.decompose(w, 4, 5)
+    idx = [0, 1, m - 5, m - 4, m - 3, m - 2, m - 1]
+    sub = kd.decompose(w[idx[0]:idx[0] + 2].contiguous(), 4, 5)
+    tail = kd.decompose(w[m - 5:].contiguous(), 4, 5)      # pairs (m-5, m-4), (m-3, m-2), (m-1)
+    torch.cuda.synchronize()
+    assert torch.equal(full.codes_u[:2], sub.codes_u) and torch.equal(full.centres_v[:2], sub.centres_v)
+    assert torch.equal(full.codes_u[m - 5:], tail.codes_u) and torch.equal(full.codes_v[m - 5:], tail.codes_v)
+    assert torch.equal(full.centres_u[m - 5:], tail.centres_u)
+    del w, full
+    # m = 0: nothing to do, no error
+    e = torch.empty((0, n), dtype=torch.float16, device="cuda")
+    out = kd.decompose(e, 4, 5)
+    assert out.codes_u.shape == (0, n // 16)
+    bat = kd.decompose_batch([e, e], 4, [1, 2])
+    assert len(bat) == 2
