@@ -118,7 +118,10 @@ def test_single_vector(kd, torch_mod):
     rep.check()
 
 
-def test_zero_and_sparse_vectors(kd, torch_mod):
+@pytest.mark.parametrize("kiters", [0, 3])
+def test_zero_and_sparse_vectors(kd, torch_mod, kiters):
+    """Degenerate vectors; with k-means on, the spike and constant vectors leave
+    clusters empty (an empty cluster keeps its centre)."""
     torch = torch_mod
     G = _rand(torch, (6, 256), seed=4)
     G[1] = 0.0                           # all-zero vector
@@ -126,7 +129,7 @@ def test_zero_and_sparse_vectors(kd, torch_mod):
     G[3, :] = 0.0
     G[3, 17] = 0.5                       # a single spike
     G[4] = 1e-3                          # constant vector
-    rep, dev = _parity(kd, torch, G, seed=5)
+    rep, dev = _parity(kd, torch, G, seed=5, kmeans_iters=kiters)
     rep.check(code_budget=False)   # the constant and spike vectors sit on boundaries by construction
     assert not dev["u"][1].any() and not dev["vhat"][1].any()
     assert not dev["centres_u"][1].any()
