@@ -710,6 +710,17 @@ def run_profile_case(args) -> None:
     layer_fn = _workloads()[args.workload][1]
     spec = dataclasses.replace(layer_fn(0)[args.profile_matrix], M=args.profile_m)
     w = synth.generate(spec, device="cuda")
+    if args.profile_kernel in ("reconstruct", "dequantise"):
+        dec = kd.decompose(w, args.iters, spec.sign_seed)
+        y = torch.empty(w.shape, dtype=torch.float16, device="cuda")
+        for _ in range(3):
+            if args.profile_kernel == "reconstruct":
+                kd.reconstruct(dec, spec.N, spec.sign_seed, dtype=torch.float16, out=y)
+            else:
+                kd.dequantise(dec.codes_u, dec.centres_u, spec.N, out=y)
+        torch.cuda.synchronize()
+        log(f"[profile-case] ok: {args.profile_kernel} n={spec.N} m={spec.M}")
+        return
     if args.profile_kernel == "rht":
         y = torch.empty(w.shape, dtype=torch.float32, device="cuda")
         for _ in range(3):
@@ -745,7 +756,7 @@ def main():
     ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
     ap.add_argument("--profile-m", type=int, default=32768)
     ap.add_argument("--profile-matrix", type=int, default=0, help="layer matrix index (0 = q, 6 = down)")
-    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht"])
+    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht", "reconstruct", "dequantise"])
     args = ap.parse_args()
     if args.profile_case:
         run_profile_case(args)
