@@ -32,6 +32,7 @@ import hashlib
 import json
 import math
 import os
+import re
 import subprocess
 import sys
 import tempfile
@@ -103,13 +104,21 @@ def fft_flops_per_vector(n: int, iters: int) -> float:
     return iters * (4 * 2.5 * n * math.log2(n) + 20 * n)
 
 
+def _code_only(text: str) -> str:
+    """C++ source without comments and blank space: edits to comments do not
+    change the kernel the profile figures were taken from."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
 def kernel_source_hash() -> str:
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2609_11687_gb300", "csrc")
     for name in DECOMPOSE_SOURCES:
-        with open(os.path.join(csrc, name), "rb") as f:
+        with open(os.path.join(csrc, name)) as f:
             h.update(name.encode())
-            h.update(f.read())
+            h.update(_code_only(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -22,9 +22,11 @@
 // Data layout per team: the spatial vector lives in registers, E = R0 complex
 // values per thread at positions t + j*T (which is exactly the first radix
 // pass's group), and a padded shared-memory buffer of N float2 carries the
-// exchanges between radix passes.  The factor u lives in registers (small E) or
-// in a per-team slot of the workspace (large N).  vhat is not stored during the
-// loop: after the last block it is recovered as P(x - u - r) (P^2 = I).
+// exchanges between radix passes.  The factor u lives in registers (the smallest
+// plans), in shared memory after the team's buffer (up to n = 11008), or in a
+// per-team slot of the workspace (n = 14336, 16384); the last two are updated in
+// place by each u-step.  vhat is not stored during the loop: after the last block
+// it is recovered as P(x - u - r) (P^2 = I).
 #pragma once
 
 #include <cstdint>
