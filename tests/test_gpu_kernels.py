@@ -271,3 +271,29 @@ def test_config2_layer0_all_vectors(kd, torch_mod, mi):
     rep, _ = _parity(kd, torch, G, spec.sign_seed)
     print(spec.name, rep)
     rep.check()
+
+
+def test_calls_only_enqueue_on_the_given_stream(kd, torch_mod):
+    """The C ABI validates, enqueues on the caller's stream and returns: right after
+    the call the stream's work (a ~4 ms decomposition) is still pending, and the
+    results are there once that stream is synchronised."""
+    torch = torch_mod
+    from paper_2609_11687_gb300 import synth
+    spec = synth.llama7b_layer(0)[4]                      # 11008 vectors of n = 4096
+    w = synth.generate(spec, device="cuda")
+    ws = kd.Workspace(spec.N)
+    ref = kd.decompose(w, ITERS, spec.sign_seed, workspace=ws)
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    out = kd.Decomposed(codes_u=torch.zeros_like(ref.codes_u), codes_v=torch.zeros_like(ref.codes_v),
+                        centres_u=torch.zeros_like(ref.centres_u), centres_v=torch.zeros_like(ref.centres_v),
+                        coeffs=None, u=None, vhat=None, resid=None, trace=None)
+    ws2 = kd.Workspace(spec.N)
+    torch.cuda.synchronize()
+    kd.decompose(w, ITERS, spec.sign_seed, workspace=ws2, out=out, stream=s)
+    done = torch.cuda.Event()
+    done.record(s)
+    assert not done.query()          # still running: the call did not wait for it
+    s.synchronize()
+    assert done.query()
+    assert torch.equal(out.codes_u, ref.codes_u) and torch.equal(out.centres_v, ref.centres_v)
