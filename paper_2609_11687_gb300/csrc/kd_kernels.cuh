@@ -491,10 +491,14 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
     };
     {
       for (int it = 0; it < p.kmeans_iters; ++it) {
-        // one factor at a time (keeps 16 accumulators live, not 32)
+        // one factor at a time.  Per vector c the thread accumulates, for each of the
+        // three boundaries b_q, the sum and count of its values above b_q, plus the
+        // total sum: cluster q holds the values above exactly q boundaries (ties
+        // low, as the codes), so the per-cluster sums and counts are differences of
+        // these -- 3 compare/select/add triples per value instead of 4.
 #pragma unroll
         for (int f = 0; f < 2; ++f) {
-          // per-thread sums [0, 8) and counts [8, 16) per (vector, centre)
+          // [c*8 + q]: sum above b_q; [c*8 + 3 + q]: count above b_q; [c*8 + 6]: total
           float acc[16];
 #pragma unroll
           for (int i = 0; i < 16; ++i) acc[i] = 0.f;
@@ -503,18 +507,18 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
 #pragma unroll
             for (int c = 0; c < 2; ++c) {
               const float x = val(j, f, c);
-              const int q = code_of(x, bnd[f][c]);
               if constexpr (TRACE) {
                 if (tracing && (c == 0 || hasB)) {
                   const int nat = nat_of<N>(lt + j * T);
-                  (c ? trB : trA)[(int64_t)(4 * p.iters + 2 * it + f) * N + nat] = (int8_t)q;
+                  (c ? trB : trA)[(int64_t)(4 * p.iters + 2 * it + f) * N + nat] = (int8_t)code_of(x, bnd[f][c]);
                 }
               }
+              acc[c * 8 + 6] = __fadd_rn(acc[c * 8 + 6], x);
 #pragma unroll
-              for (int qq = 0; qq < 4; ++qq) {
-                const bool hit = (q == qq);
-                acc[c * 4 + qq] = __fadd_rn(acc[c * 4 + qq], hit ? x : 0.f);
-                acc[8 + c * 4 + qq] = __fadd_rn(acc[8 + c * 4 + qq], hit ? 1.f : 0.f);
+              for (int q = 0; q < 3; ++q) {
+                const bool gt = x > bnd[f][c][q];
+                acc[c * 8 + q] = __fadd_rn(acc[c * 8 + q], gt ? x : 0.f);
+                acc[c * 8 + 3 + q] = __fadd_rn(acc[c * 8 + 3 + q], gt ? 1.f : 0.f);
               }
             }
           }
@@ -522,10 +526,13 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
           team_sum_k<PL, 16>(acc, tot, reinterpret_cast<float*>(red), lt);
 #pragma unroll
           for (int c = 0; c < 2; ++c) {
+            const float* t = tot + c * 8;
+            // counts are exact integers in fp32 (n <= 16384)
+            const float sum[4] = {__fsub_rn(t[6], t[0]), __fsub_rn(t[0], t[1]), __fsub_rn(t[1], t[2]), t[2]};
+            const float cnt[4] = {__fsub_rn((float)N, t[3]), __fsub_rn(t[3], t[4]), __fsub_rn(t[4], t[5]), t[5]};
 #pragma unroll
             for (int qq = 0; qq < 4; ++qq) {
-              const float n_ = tot[8 + c * 4 + qq];
-              if (n_ > 0.f) cen[f][c][qq] = __fdiv_rn(tot[c * 4 + qq], n_);
+              if (cnt[qq] > 0.f) cen[f][c][qq] = __fdiv_rn(sum[qq], cnt[qq]);
             }
 #pragma unroll
             for (int qq = 0; qq < 3; ++qq)
