@@ -395,9 +395,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         }
         team_sync<PL>();  // the last transform's readers of buf are done
       } else if ((hb & 1) == 0) {
-        // two greedy steps from Q_N (update u)
-        float2 l1 = make_float2(0.f, 0.f);
-        // u outside registers (shared memory, or the workspace slot for the longest
+        // two greedy steps from Q_N (update u).  u outside registers (shared memory, or the workspace slot for the longest
         // vectors) is updated in place by both steps: two roundings, as with two
         // separate updates
         auto add_slot = [&](int j, float dA, float dB) {
@@ -410,7 +408,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
             uslot[lt + j * T] = uj;
           }
         };
-        l1 = greedy(step, hb == 0, sum0, add_slot);
+        const float2 l1 = greedy(step, hb == 0, sum0, add_slot);
         ++step;
         const float2 l2 = greedy(step, false, sum0, add_slot);
         ++step;
