@@ -395,9 +395,9 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
         }
         team_sync<PL>();  // the last transform's readers of buf are done
       } else if ((hb & 1) == 0) {
-        // two greedy steps from Q_N (update u).  u outside registers (shared memory, or the workspace slot for the longest
-        // vectors) is updated in place by both steps: two roundings, as with two
-        // separate updates
+        // two greedy steps from Q_N (update u).  u outside registers (shared memory,
+        // or the workspace slot for the longest vectors) is updated in place by both
+        // steps: two roundings, as with two separate updates
         auto add_slot = [&](int j, float dA, float dB) {
           if constexpr (PL::UMODE == UREG) {
             add_u(j, dA, dB);
