@@ -34,9 +34,14 @@
  *              nothing is enqueued; a failed launch returns KD_ERR_CUDA; a
  *              non-finite input value is detected on the device and reported
  *              by kd_read_status().  No call traps or aborts.
- *  Supported n: n even, 16 <= n <= 16384, with a compiled plan (kd_supported());
- *              at least 256, 512, 768, 1024, 1536, 2048, 3072, 4096, 8192,
- *              11008, 14336, 16384.
+ *  Supported n: 1 <= n <= 16384 whose prime factors all lie in
+ *              {2, 3, 5, 7, 11, 13, 43} (kd_supported()).  Sixteen lengths have a
+ *              compiled, tuned plan (kd_tuned()): 16, 32, 64, 128, 256, 512, 768,
+ *              1024, 1536, 2048, 3072, 4096, 8192, 11008, 14336, 16384.  Every other
+ *              supported length runs a run-time-length path (transform radices
+ *              chosen per call, the pair held in shared memory): same method and
+ *              outputs, several times slower.  Code words per vector: ceil(n/16),
+ *              the last one padded with zero codes.
  */
 #ifndef KASHIN_H
 #define KASHIN_H
@@ -51,7 +56,7 @@ extern "C" {
 typedef enum {
   KD_OK = 0,
   KD_ERR_INVALID_ARG = 1,   /* null required pointer, bad size, bad enum, ld too small */
-  KD_ERR_UNSUPPORTED_N = 2, /* no compiled plan for this vector length */
+  KD_ERR_UNSUPPORTED_N = 2, /* vector length outside the supported set (see "Supported n") */
   KD_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed */
   KD_ERR_NONFINITE = 4,     /* a decomposed vector held NaN or Inf (device-detected) */
   KD_ERR_WORKSPACE = 5      /* workspace pointer null or smaller than kd_workspace_size() */
@@ -67,8 +72,13 @@ const char* kd_status_string(kd_status s);
 /* Library version string. */
 const char* kd_version(void);
 
-/* KD_OK if vector length n has a compiled plan, else KD_ERR_UNSUPPORTED_N. */
+/* KD_OK if vector length n is supported (see "Supported n" above), else
+ * KD_ERR_UNSUPPORTED_N. */
 kd_status kd_supported(int64_t n);
+
+/* 1 if vector length n has a compiled, tuned plan, else 0 (unsupported lengths
+ * included).  Informational: every supported n runs through the same calls. */
+int kd_tuned(int64_t n);
 
 /* Bytes of device workspace kd_decompose / kd_apply_p / kd_reconstruct need for
  * vector length n on the current device (0 if n is unsupported).  The workspace
@@ -122,7 +132,9 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
  * synchronisation).  The paper has no counterpart: this is a library convenience.
  * Same arguments and results as kd_decompose minus workspace/ws_bytes; the scratch
  * lives in a 160 KB static device array inside the library instead.
- *   - n <= 8192 only; larger n returns KD_ERR_WORKSPACE and enqueues nothing.
+ *   - n <= 8192 whose workspace fits the array (the tuned lengths; the run-time-length
+ *     path needs per-CTA slots that do not fit); otherwise KD_ERR_WORKSPACE and
+ *     nothing is enqueued.
  *   - Allocates nothing.  Every GPU that loads the library holds the array until exit.
  *   - All calls share the array (it keeps the last call's tables); each call rewrites
  *     what it needs on its own stream, so calls that overlap on the GPU race.
@@ -142,8 +154,9 @@ kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, i
  * CTAs, so small matrices fill the GPU and the last wave of one matrix overlaps the
  * next.  Each matrix keeps its own sign seed, leading dimension and outputs; the
  * arithmetic per vector pair is identical to kd_decompose's (bitwise equal results).
- * Lengths n <= 8192 run as one launch; longer vectors (which fill the GPU alone)
- * run one launch per matrix, in order, on the same stream and workspace.
+ * Tuned lengths n <= 8192 run as one launch; longer vectors (which fill the GPU
+ * alone) and the run-time-length path run one launch per matrix, in order, on the
+ * same stream and workspace.
  *
  *   mats      HOST array of `count` descriptors (1 <= count <= KD_MAX_BATCH); read
  *             during the call only.  In each: w, m, ld, sign_seed as kd_decompose's

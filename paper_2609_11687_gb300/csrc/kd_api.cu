@@ -13,7 +13,7 @@ KD_PLAN(1024) KD_PLAN(1536) KD_PLAN(2048) KD_PLAN(3072) KD_PLAN(4096) KD_PLAN(81
 KD_PLAN(11008) KD_PLAN(14336) KD_PLAN(16384)
 #undef KD_PLAN
 
-const PlanOps* plan_ops(int64_t n) {
+const PlanOps* tuned_plan_ops(int64_t n) {
   switch (n) {
     case 16: return plan_ops_16();
     case 32: return plan_ops_32();
@@ -33,6 +33,11 @@ const PlanOps* plan_ops(int64_t n) {
     case 16384: return plan_ops_16384();
     default: return nullptr;
   }
+}
+
+const PlanOps* plan_ops(int64_t n) {
+  const PlanOps* ops = tuned_plan_ops(n);
+  return ops ? ops : generic_plan_ops(n);
 }
 
 namespace {
@@ -75,7 +80,7 @@ int sm_count() {
 
 // Most CTAs a decompose launch of this plan ever uses on the current device.
 int max_decompose_ctas(const PlanOps* ops) {
-  const int per = ops->ctas_per_sm(0);
+  const int per = ops->ctas_per_sm(0, ops->n);
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return 0;
   return per * sms;
@@ -100,7 +105,7 @@ bool layout_of(const PlanOps* ops, WsLayout* L, int nsets = 1) {
 kd_status setup(const PlanOps* ops, const WsLayout& L, void* ws, uint64_t seed, cudaStream_t s) {
   char* b = static_cast<char*>(ws);
   cudaError_t e = ops->setup(reinterpret_cast<float2*>(b + L.tw), reinterpret_cast<uint32_t*>(b + L.eps),
-                             reinterpret_cast<uint32_t*>(b + L.status), seed, s);
+                             reinterpret_cast<uint32_t*>(b + L.status), seed, ops->n, s);
   return e == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
@@ -134,6 +139,8 @@ const char* kd_status_string(kd_status s) {
 const char* kd_version(void) { return "libkashin 0.1.0 (sm_103a)"; }
 
 kd_status kd_supported(int64_t n) { return plan_ops(n) ? KD_OK : KD_ERR_UNSUPPORTED_N; }
+
+int kd_tuned(int64_t n) { return tuned_plan_ops(n) ? 1 : 0; }
 
 size_t kd_workspace_size(int64_t n) {
   const PlanOps* ops = plan_ops(n);
@@ -303,11 +310,12 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
   ApplyParams p;
   p.x = x;
   p.y = y;
+  p.n = n;
   p.m = m;
   p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.npairs = (m + 1) / 2;
-  const int per = ops->ctas_per_sm(1);
+  const int per = ops->ctas_per_sm(1, n);
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, per * sms);
@@ -339,13 +347,14 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
   p.codes_v = codes_v;
   p.centres_u = centres_u;
   p.centres_v = centres_v;
+  p.n = n;
   p.m = m;
   p.ld = ld;
   p.out = w_hat;
   p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.npairs = (m + 1) / 2;
-  const int per = ops->ctas_per_sm(2);
+  const int per = ops->ctas_per_sm(2, n);
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, per * sms);

@@ -606,7 +606,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
 struct ApplyParams {
   const float* x;
   float* y;
-  int64_t m;
+  int64_t n, m;
   const float2* twt;
   const uint32_t* eps;
   int64_t npairs;
@@ -659,7 +659,7 @@ struct RecParams {
   const uint32_t* codes_v;
   const float* centres_u;
   const float* centres_v;
-  int64_t m, ld;
+  int64_t n, m, ld;
   void* out;
   const float2* twt;
   const uint32_t* eps;

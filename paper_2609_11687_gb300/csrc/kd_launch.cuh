@@ -50,14 +50,14 @@ struct Ops {
     k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
     return cudaGetLastError();
   }
-  static cudaError_t setup(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, cudaStream_t s) {
+  static cudaError_t setup(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, int64_t, cudaStream_t s) {
     constexpr int threads = 256;
     constexpr int work = PL::TWN > (PL::N + 31) / 32 ? PL::TWN : (PL::N + 31) / 32;
     constexpr int blocks = (work + threads - 1) / threads;
     setup_kernel<PL><<<blocks, threads, 0, s>>>(twt, eps, status, seed);
     return cudaGetLastError();
   }
-  static int ctas_per_sm(int which) {
+  static int ctas_per_sm(int which, int64_t) {
     if (which == 0) return occupancy(decompose_kernel<PL, false>, PL::THREADS, PL::SMEM);
     if (which == 1) return occupancy(apply_p_kernel<PL>, PL::THREADS, PL::SMEM);
     return occupancy(reconstruct_kernel<PL>, PL::THREADS, PL::SMEM);

@@ -29,7 +29,7 @@ KD_OK, KD_ERR_INVALID_ARG, KD_ERR_UNSUPPORTED_N, KD_ERR_CUDA, KD_ERR_NONFINITE, 
 KD_F32, KD_F16, KD_BF16 = 0, 1, 2
 KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
-EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_workspace_size", "kd_signs",
+EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_measure_fp32_peak", "kd_workspace_size_batch",
            "kd_decompose_batch")
@@ -55,6 +55,8 @@ def _load() -> ctypes.CDLL:
     lib.kd_version.restype = ctypes.c_char_p
     lib.kd_supported.argtypes = [c_i64]
     lib.kd_supported.restype = c_int
+    lib.kd_tuned.argtypes = [c_i64]
+    lib.kd_tuned.restype = c_int
     lib.kd_workspace_size.argtypes = [c_i64]
     lib.kd_workspace_size.restype = c_sz
     lib.kd_signs.argtypes = [c_u64, c_i64, c_vp]
@@ -109,6 +111,10 @@ def kd_supported(n: int) -> int:
     return lib.kd_supported(int(n))
 
 
+def kd_tuned(n: int) -> bool:
+    return bool(lib.kd_tuned(int(n)))
+
+
 def kd_workspace_size(n: int) -> int:
     return int(lib.kd_workspace_size(int(n)))
 
@@ -142,8 +148,9 @@ def kd_reconstruct(codes_u, codes_v, centres_u, centres_v, n, m, sign_seed, out_
 
 def kd_batchable(n: int) -> bool:
     """True when kd_decompose_batch runs all matrices of length n in one launch
-    (n <= 8192, as include/kashin.h states); longer vectors run one launch each."""
-    return kd_supported(n) == KD_OK and int(n) <= 8192
+    (tuned lengths n <= 8192, as include/kashin.h states); longer vectors and the
+    run-time-length path run one launch each."""
+    return kd_tuned(n) and int(n) <= 8192
 
 
 def kd_workspace_size_batch(n: int, count: int) -> int:

@@ -55,11 +55,33 @@ def test_kd_signs_match_oracle(kd, seed, n):
     np.testing.assert_array_equal(kd.kd_signs(seed, n), ko.sign_mask(seed, n).astype(np.int8))
 
 
+TUNED = (16, 32, 64, 128, 256, 512, 768, 1024, 1536, 2048, 3072, 4096, 8192, 11008, 14336, 16384)
+
+
+def _smooth(n):
+    """1 <= n <= 16384 with every prime factor in {2, 3, 5, 7, 11, 13, 43}."""
+    if n < 1 or n > 16384:
+        return False
+    for p in (2, 3, 5, 7, 11, 13, 43):
+        while n % p == 0:
+            n //= p
+    return n == 1
+
+
 def test_supported_lengths(kd):
-    for n in (16, 256, 768, 3072, 4096, 11008, 14336, 16384):
-        assert kd.kd_supported(n) == kd.KD_OK
-    for n in (0, 1, 15, 100, 4095, 32768):
-        assert kd.kd_supported(n) == kd.KD_ERR_UNSUPPORTED_N
+    for n in TUNED:
+        assert kd.kd_supported(n) == kd.KD_OK and kd.kd_tuned(n)
+    # the run-time-length path: every other length whose prime factors are in the set
+    for n in (1, 2, 3, 15, 43, 100, 2560, 4095, 5120, 13824, 16000):
+        assert kd.kd_supported(n) == kd.KD_OK and not kd.kd_tuned(n)
+    for n in (0, -16, 17, 4094, 16385, 32768):
+        assert kd.kd_supported(n) == kd.KD_ERR_UNSUPPORTED_N and not kd.kd_tuned(n)
+
+
+def test_supported_set_is_the_factor_rule(kd):
+    got = [n for n in range(0, 16400) if kd.kd_supported(n) == kd.KD_OK]
+    assert got == [n for n in range(0, 16400) if _smooth(n)]
+    assert [n for n in range(0, 16400) if kd.kd_tuned(n)] == list(TUNED)
 
 
 def test_workspace_size_register_plans(kd):
@@ -67,13 +89,13 @@ def test_workspace_size_register_plans(kd):
     for n in (256, 768, 4096):
         ws = kd.kd_workspace_size(n)
         assert ws >= 256 + 8 * n + n // 8 and ws % 256 == 0   # status, sign bits, pass-0 twiddles
-    assert kd.kd_workspace_size(100) == 0
+    assert kd.kd_workspace_size(4094) == 0
 
 
 def test_argument_validation_without_gpu(kd):
     null = None
     # unsupported length
-    st = kd.kd_decompose(1, 0, 0, 100, 4, 100, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20, null)
+    st = kd.kd_decompose(1, 0, 0, 4094, 4, 4094, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20, null)
     assert st == kd.KD_ERR_UNSUPPORTED_N
     # out-of-range refinement count
     assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 65, 1, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
@@ -129,7 +151,7 @@ def test_batch_workspace_and_validation(kd):
         big = kd.kd_workspace_size_batch(n, 32)
         assert big > one and big >= 256 + 32 * (n // 8) + 8 * n   # status, 32 sign sets, twiddles
     assert kd.kd_workspace_size_batch(4096, 0) == 0 and kd.kd_workspace_size_batch(4096, 33) == 0
-    assert kd.kd_workspace_size_batch(100, 2) == 0
+    assert kd.kd_workspace_size_batch(4094, 2) == 0
     arr = (kd.KdMatrix * 2)()
     for i in range(2):
         arr[i] = kd.KdMatrix(None, 0, 4096, i, None, None, None, None, None)
@@ -138,7 +160,7 @@ def test_batch_workspace_and_validation(kd):
     assert kd.kd_decompose_batch(ptr, 0, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_decompose_batch(ptr, 33, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_decompose_batch(null, 2, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
-    assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4095, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_UNSUPPORTED_N
+    assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4094, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_UNSUPPORTED_N
     assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4096, 4, 0, 1, 16, null) == kd.KD_ERR_WORKSPACE
     arr[1] = kd.KdMatrix(None, 3, 4096, 1, None, None, None, None, None)   # m > 0 without pointers
     assert kd.kd_decompose_batch(ptr, 2, 0, 0, 4096, 4, 0, 1, 1 << 30, null) == kd.KD_ERR_INVALID_ARG
