@@ -216,6 +216,14 @@ struct Xform {
   Mask ek, em;                 // eps_k < 0 / eps_{-k} < 0 for each owned frequency (bit index)
   Mask dm;                     // ek ^ em: frequencies whose M takes the partner value
   static constexpr float kInvN = 1.0f / (float)N;
+  // Warp-local middle passes (16 x 16 x 16 with 256 threads): after pass 0 the
+  // vector falls into 16 blocks of 256 slots (one per pass-0 output digit b), and the
+  // M partner of every last-pass group of block b lies in block 16 - b (blocks 0 and
+  // 8 pair with themselves).  Warp w owns blocks {w, 16 - w} ({0, 8} for w = 0) for
+  // pass 1, the last pass and the inverse pass 1, so only the exchanges into and
+  // out of pass 0 cross warps: two CTA barriers per P instead of four.
+  static constexpr bool WL = NP == 3 && PL::PAIRED && E == 16 && PL::R(1) == 16 && PL::RL == 16 && T == 256;
+  int g1;                      // warp-local: this thread's pass-1 group
   int p0, p1;                  // slot-order M: partner slot constants
   int pb0;                     // pad(lt): base of the pass-0 slots lt + j T
   int pbp0, pbp1;              // slot-order M: pad(p0), pad(p1)
@@ -232,7 +240,18 @@ struct Xform {
       constexpr int H = PL::HALF;
       constexpr int L = T;
       const int w = lt / (2 * H), l = lt % (2 * H), h = l / H, i = l % H;
-      const int bb = H * w + i;
+      // partner groups K and T - K at lanes l and l ^ H (K = 0 and T/2 pair with
+      // themselves, at lanes 0 and H of warp 0)
+      int bb;
+      if constexpr (WL) {
+        // last-pass group K = b + 16 k1 (b: pass-0 digit = block, k1: pass-1 digit);
+        // warp w >= 1 holds blocks w and 16 - w, warp 0 blocks 0 and 8
+        bb = (w == 0) ? (i < 8 ? 16 * i : 16 * i - 120) : w + 16 * i;
+        g1 = ((w == 0) ? 8 * h : (h ? 16 - w : w)) * 16 + i;
+      } else {
+        bb = H * w + i;
+        g1 = 0;
+      }
       kgrp = h ? (bb ? L - bb : L / 2) : bb;
       self = (bb == 0) ? (h == 0 ? 1 : 2) : 0;
       lbase = slot_low<PL>(kgrp);
@@ -245,7 +264,7 @@ struct Xform {
       pbp0 = pad(p0);
       pbp1 = pad(p1);
       cw = expi_pi((long long)E * Kp, N);
-      kgrp = self = lbase = 0;
+      kgrp = self = lbase = g1 = 0;
     }
     set_eps(eb);
   }
@@ -348,7 +367,9 @@ struct Xform {
     constexpr bool LAST = (I == NP - 1);
     constexpr int OFF = PL::tw_off(I);
     constexpr bool SEP = PL::sep_pass(I);
-    for (int g = lt; g < G; g += T) {
+    // warp-local plans: pass 1 has one group per thread, in one of the warp's blocks
+    constexpr bool ONE = WL && I == 1;
+    for (int g = ONE ? g1 : lt; ONE || g < G; g += T) {
       const int blk = g / S;
       const int np = g - blk * S;
       const int base = blk * Bk + np;
@@ -372,6 +393,7 @@ struct Xform {
       }
 #pragma unroll
       for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
+      if constexpr (ONE) break;
     }
   }
 
@@ -439,10 +461,12 @@ struct Xform {
     if constexpr (PL::PAIRED) {
       static_for<1, NP - 1>([&](auto ii) {
         pass<decltype(ii)::value, -1>();
-        team_sync<PL>();
+        if constexpr (WL) __syncwarp();
+        else team_sync<PL>();
       });
       last_paired();
-      team_sync<PL>();
+      if constexpr (WL) __syncwarp();
+      else team_sync<PL>();
       static_for<1, NP - 1>([&](auto ii) {
         pass<NP - 1 - decltype(ii)::value, +1>();
         team_sync<PL>();

@@ -1,5 +1,6 @@
-"""Fig. 2's properties on the device path: Gaussian vectors at the supported
-lengths nearest the figure's N = 10^4 (11008, 16384) and one below it (8192).
+"""Fig. 2's properties on the device path: Gaussian vectors at the figure's own
+N = 10^4 (2^4 5^4, the run-time-length path) and at the compiled lengths around
+it (8192, 11008, 16384).
 Algorithm 1 on the GPU must leave both factors on four sharp peaks (best
 four-level distortion far below a Gaussian's 0.1175), and the device's k-means
 refinement must converge to the Lloyd optimum near the closed-form centres."""
@@ -25,7 +26,7 @@ def kd():
     return kashin
 
 
-@pytest.mark.parametrize("n", [8192, 11008, 16384])
+@pytest.mark.parametrize("n", [8192, 10000, 11008, 16384])
 def test_gpu_fig2_four_peaks_and_lloyd(kd, n):
     import torch
     m = 4
