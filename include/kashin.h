@@ -59,7 +59,7 @@ typedef enum {
   KD_ERR_UNSUPPORTED_N = 2, /* vector length outside the supported set (see "Supported n") */
   KD_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed */
   KD_ERR_NONFINITE = 4,     /* a decomposed vector held NaN or Inf (device-detected) */
-  KD_ERR_WORKSPACE = 5      /* workspace pointer null or smaller than kd_workspace_size() */
+  KD_ERR_WORKSPACE = 5      /* workspace pointer null, not 16-byte aligned, or too small */
 } kd_status;
 
 typedef enum { KD_F32 = 0, KD_F16 = 1, KD_BF16 = 2 } kd_dtype;
@@ -116,7 +116,8 @@ kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host);
  *             order); rows 4k + 2t + f hold the cluster (0..3) of factor f (0 = u,
  *             1 = vhat) in refinement iteration t.  Test/debug output; enabling it
  *             does not change any other output bit.
- *  workspace  device scratch of ws_bytes >= kd_workspace_size(n).
+ *  workspace  device scratch, 16-byte aligned (as cudaMalloc returns), of
+ *             ws_bytes >= kd_workspace_size(n).
  *
  * Vectors are processed two at a time (2j, 2j+1); each vector's results depend
  * only on its own data and its pair partner's (through rounding only). */

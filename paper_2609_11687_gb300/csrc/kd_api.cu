@@ -45,6 +45,10 @@ namespace {
 constexpr size_t kAlign = 256;
 inline size_t align_up(size_t x) { return (x + kAlign - 1) / kAlign * kAlign; }
 
+// A workspace must be non-null and 16-byte aligned (its tables are read with
+// 128-bit loads); cudaMalloc and the caching allocators return 256-byte alignment.
+inline bool ws_ok(const void* ws) { return ws && reinterpret_cast<uintptr_t>(ws) % 16 == 0; }
+
 // Workspace layout: [status word | pad][sign bits, one set per matrix][access-ordered twiddles][u slots]
 struct WsLayout {
   size_t status, eps, tw, uslots, total;
@@ -175,7 +179,7 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
   if (m > 0 && (!w || !codes_u || !codes_v || !centres_u || !centres_v)) return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
-  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   kd_status st = setup(ops, L, workspace, sign_seed, s);
   if (st != KD_OK || m == 0) return st;
@@ -246,7 +250,7 @@ kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, k
   }
   WsLayout L;
   if (!layout_of(ops, &L, count)) return KD_ERR_CUDA;
-  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   if (!ops->batch) {
     // long vectors: one launch per matrix on the same workspace, in stream order
@@ -302,7 +306,7 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
   if (m > 0 && (!x || !y)) return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
-  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   kd_status st = setup(ops, L, workspace, sign_seed, s);
   if (st != KD_OK || m == 0) return st;
@@ -335,7 +339,7 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
     return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
-  if (!workspace || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   kd_status st = setup(ops, L, workspace, sign_seed, s);
   if (st != KD_OK || m == 0) return st;
@@ -362,7 +366,7 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
 }
 
 kd_status kd_read_status(const void* workspace, void* stream) {
-  if (!workspace) return KD_ERR_WORKSPACE;
+  if (!ws_ok(workspace)) return KD_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   uint32_t word = 0;
   if (cudaMemcpyAsync(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess) return KD_ERR_CUDA;

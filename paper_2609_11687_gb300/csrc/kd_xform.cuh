@@ -69,6 +69,21 @@ __device__ __forceinline__ float2 ld_tw(const float2* p) {
 
 
 
+// Two consecutive table entries (16-byte aligned) in one 128-bit load.
+template <bool SMEM>
+__device__ __forceinline__ float4 ld_tw4(const float2* p) {
+  float4 v;
+  if constexpr (SMEM) {
+    const unsigned a = (unsigned)__cvta_generic_to_shared(p);
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
+  } else {
+    asm volatile("ld.global.nc.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "l"(p));
+  }
+  return v;
+}
+
 template <int N_, int T_, int Q_, int UMODE_, int MINB_, int... Rs>
 struct Plan {
   static constexpr int N = N_;
@@ -108,10 +123,24 @@ struct Plan {
     return o;
   }
   static constexpr int TWN = tw_off(NP - 1);
+
   // stage the table in shared memory when MINB CTAs per SM still fit
   static constexpr int TEAM = BUF + RED + USL;  // float2 slots of shared memory per team
   static constexpr bool TW_SMEM = (size_t)TWN * 8 + (size_t)Q * TEAM * 8 <= (size_t)(227 * 1024) / MINB - 1024;
   static constexpr size_t SMEM_TW = TW_SMEM ? (size_t)TWN * sizeof(float2) : 0;
+  // paired twiddle layout (table staged in shared memory, every twiddled pass of even
+  // radix): rows 2a and 2a + 1 of a pass table are interleaved per column
+  // ([a][column][2]), so one 128-bit load fetches a column's twiddles of both rows
+  KD_HD static constexpr bool tw2_ok() {
+    for (int i = 0; i < NP - 1; ++i)
+      if (Rv[i] % 2 != 0) return false;
+    return TW_SMEM;
+  }
+  static constexpr bool TW2 = tw2_ok();
+  // table position of row j, column c of pass i (rows of length L)
+  KD_HD static constexpr int tw_pos(int i, int L, int j, int c) {
+    return tw_off(i) + (TW2 ? (j / 2) * 2 * L + 2 * c + (j % 2) : j * L + c);
+  }
   static constexpr size_t SMEM = SMEM_TW + (size_t)Q * TEAM * sizeof(float2);
 
   // pass 0 / inverse pass 0 and slot-order M: slots base + j*T with base < T
@@ -313,23 +342,46 @@ struct Xform {
     return __fmul2_rn(sel, make_float2(f, f));
   }
 
+  // v[j] *= W (DIR < 0) or conj(W) (DIR > 0) for j = 1 .. R-1, W = the entry (j, c)
+  // of pass I's twiddle table (rows of length L)
+  template <int I, int L, int R, int DIR>
+  __device__ __forceinline__ void twiddle(float2 (&v)[R], int c) const {
+    auto mul = [](float2 a, float2 w) { return DIR < 0 ? cmul(a, w) : cmulc(a, w); };
+    if constexpr (PL::TW2) {
+      static_assert(R % 2 == 0, "paired twiddles need an even radix");
+      static_for<0, R / 2>([&](auto pc) {
+        constexpr int P = decltype(pc)::value;
+        constexpr int O = PL::tw_pos(I, L, 2 * P, 0);
+        const float2* q = tw + O + 2 * c;
+        if constexpr (P == 0) {
+          v[1] = mul(v[1], ld_tw<PL::TW_SMEM>(q + 1));
+        } else {
+          const float4 w = ld_tw4<PL::TW_SMEM>(q);
+          v[2 * P] = mul(v[2 * P], make_float2(w.x, w.y));
+          v[2 * P + 1] = mul(v[2 * P + 1], make_float2(w.z, w.w));
+        }
+      });
+    } else {
+      constexpr int O = PL::tw_off(I);
+#pragma unroll
+      for (int j = 1; j < R; ++j) v[j] = mul(v[j], ld_tw<PL::TW_SMEM>(tw + O + j * L + c));
+    }
+  }
+
   // forward pass 0 from registers
   __device__ __forceinline__ void fwd0(float2 (&v)[E]) {
     if constexpr (kd_is_big_prime<E>()) {
+      static_assert(!PL::TW2, "row-major pass-0 table");
       dft_prime_stream<E, -1>([&](auto jc) { return v[decltype(jc)::value]; },
                               [&](auto kc, float2 x) {
                                 constexpr int K = decltype(kc)::value;
-                                if constexpr (K > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + K * T + lt));
+                                if constexpr (K > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + K * T + lt));  // row-major: E odd
                                 buf[a0<K>()] = x;
                               });
     } else {
       Dft<E, -1>::run(v);
-      static_for<0, E>([&](auto jc) {
-        constexpr int J = decltype(jc)::value;
-        float2 x = v[J];
-        if constexpr (J > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));
-        buf[a0<J>()] = x;
-      });
+      twiddle<0, T, E, -1>(v, lt);
+      static_for<0, E>([&](auto jc) { buf[a0<decltype(jc)::value>()] = v[decltype(jc)::value]; });
     }
   }
 
@@ -341,18 +393,14 @@ struct Xform {
           [&](auto jc) {
             constexpr int J = decltype(jc)::value;
             float2 x = buf[a0<J>()];
-            if constexpr (J > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));
+            if constexpr (J > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));  // row-major: E odd
             return x;
           },
           [&](auto kc, float2 x) { buf[a0<decltype(kc)::value>()] = x; });
       static_for<0, E>([&](auto jc) { v[decltype(jc)::value] = buf[a0<decltype(jc)::value>()]; });
     } else {
-      static_for<0, E>([&](auto jc) {
-        constexpr int J = decltype(jc)::value;
-        float2 x = buf[a0<J>()];
-        if constexpr (J > 0) x = cmulc(x, ld_tw<PL::TW_SMEM>(tw + J * T + lt));
-        v[J] = x;
-      });
+      static_for<0, E>([&](auto jc) { v[decltype(jc)::value] = buf[a0<decltype(jc)::value>()]; });
+      twiddle<0, T, E, +1>(v, lt);
       Dft<E, +1>::run(v);
     }
   }
@@ -380,15 +428,9 @@ struct Xform {
       for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
       if constexpr (DIR < 0) {
         Dft<R, -1>::run(v);
-        if constexpr (!LAST) {
-#pragma unroll
-          for (int j = 1; j < R; ++j) v[j] = cmul(v[j], ld_tw<PL::TW_SMEM>(tw + OFF + j * S + np));
-        }
+        if constexpr (!LAST) twiddle<I, S, R, -1>(v, np);
       } else {
-        if constexpr (!LAST) {
-#pragma unroll
-          for (int j = 1; j < R; ++j) v[j] = cmulc(v[j], ld_tw<PL::TW_SMEM>(tw + OFF + j * S + np));
-        }
+        if constexpr (!LAST) twiddle<I, S, R, +1>(v, np);
         Dft<R, +1>::run(v);
       }
 #pragma unroll
@@ -511,14 +553,18 @@ __global__ void setup_kernel(float2* twt, uint32_t* eps, uint32_t* status, uint6
       constexpr int LEN = PL::B(I);
       if (e >= OFF && e < OFF + LEN) {
         const int r = e - OFF;
-        if constexpr (I == 0) {  // [j][t]: W_N^{t j}
-          m = (long long)(r % PL::T) * (r / PL::T);
-          b = PL::N;
-        } else {                 // [j][np]: W_B^{np j}
-          constexpr int S = PL::S(I);
-          m = (long long)(r % S) * (r / S);
-          b = LEN;
+        // row j, column c: pass 0 W_N^{c j} (c = thread), pass I W_B^{c j} (c = np)
+        constexpr int L = (I == 0) ? PL::T : PL::S(I);
+        int j, c;
+        if constexpr (PL::TW2) {  // [j / 2][c][j % 2]
+          j = 2 * (r / (2 * L)) + (r % 2);
+          c = (r % (2 * L)) / 2;
+        } else {                  // [j][c]
+          j = r / L;
+          c = r % L;
         }
+        m = (long long)c * j;
+        b = (I == 0) ? PL::N : LEN;
       }
     });
     twt[e] = root_w(m, b);

@@ -117,6 +117,9 @@ def test_argument_validation_without_gpu(kd):
                            null) == kd.KD_ERR_WORKSPACE
     assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 16,
                            null) == kd.KD_ERR_WORKSPACE
+    # workspace not 16-byte aligned (its tables are read with 128-bit loads)
+    assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null, 8, 1 << 20,
+                           null) == kd.KD_ERR_WORKSPACE
     assert kd.kd_apply_p(1, 1, 256, 2, 0, null, 0, null) == kd.KD_ERR_WORKSPACE
     assert kd.kd_apply_p(null, 1, 256, 2, 0, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_reconstruct(1, 1, 1, 1, 256, 2, 0, 9, 0, 1, 256, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
