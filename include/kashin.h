@@ -217,6 +217,25 @@ kd_status kd_read_status(const void* workspace, void* stream);
 kd_status kd_dequantise(const uint32_t* codes, const float* centres, int64_t n, int64_t m, kd_dtype out_dtype,
                         kd_layout layout, void* out, int64_t ld, void* stream);
 
+/* kd_dequantise for several planes of one vector length n in one launch (App. C at
+ * load time: a layer's U_q and V_q planes together), so that small planes do not
+ * each pay a launch and a partly filled last wave.
+ *   planes  HOST array of `count` descriptors (1 <= count <= KD_MAX_BATCH), read
+ *           during the call; each as kd_dequantise's codes, centres, m, out and ld.
+ * Every plane is written exactly as kd_dequantise would write it; outputs that
+ * overlap give undefined contents.  Errors as kd_dequantise (the first invalid
+ * plane's), and KD_ERR_INVALID_ARG for a bad count or a null array. */
+typedef struct kd_plane {
+  const uint32_t* codes;
+  const float* centres;
+  void* out;
+  int64_t m;
+  int64_t ld;
+} kd_plane;
+
+kd_status kd_dequantise_batch(const kd_plane* planes, int count, int64_t n, kd_dtype out_dtype, kd_layout layout,
+                              void* stream);
+
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:
  * the weights are rotated by a randomized Hadamard transform before the

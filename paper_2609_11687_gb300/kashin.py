@@ -31,9 +31,15 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
-           "kd_rht_block", "kd_rht", "kd_dequantise", "kd_measure_fp32_peak", "kd_workspace_size_batch",
-           "kd_decompose_batch")
+           "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
+           "kd_workspace_size_batch", "kd_decompose_batch")
 KD_MAX_BATCH = 32
+
+
+class KdPlane(ctypes.Structure):
+    """kd_plane: one 2-bit code plane to expand (kd_dequantise_batch)."""
+    _fields_ = [("codes", ctypes.c_void_p), ("centres", ctypes.c_void_p), ("out", ctypes.c_void_p),
+                ("m", ctypes.c_int64), ("ld", ctypes.c_int64)]
 
 
 class KdMatrix(ctypes.Structure):
@@ -79,6 +85,8 @@ def _load() -> ctypes.CDLL:
     lib.kd_measure_fp32_peak.restype = c_int
     lib.kd_dequantise.argtypes = [c_vp, c_vp, c_i64, c_i64, c_int, c_int, c_vp, c_i64, c_vp]
     lib.kd_dequantise.restype = c_int
+    lib.kd_dequantise_batch.argtypes = [c_vp, c_int, c_i64, c_int, c_int, c_vp]
+    lib.kd_dequantise_batch.restype = c_int
     lib.kd_rht_block.argtypes = [c_i64]
     lib.kd_rht_block.restype = c_i64
     lib.kd_rht.argtypes = [c_vp, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_vp, c_i64, c_vp, c_vp]
@@ -167,6 +175,10 @@ def kd_read_status(workspace, stream) -> int:
 
 def kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream) -> int:
     return lib.kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream)
+
+
+def kd_dequantise_batch(planes, count, n, out_dtype, layout, stream) -> int:
+    return lib.kd_dequantise_batch(planes, count, n, out_dtype, layout, stream)
 
 
 def measure_fp32_peak(stream=None) -> float:
@@ -361,6 +373,33 @@ def dequantise(codes, centres, n: int, dtype=None, layout: str = "rows", out=Non
     if st != KD_OK:
         raise KashinError(st, "kd_dequantise")
     return out
+
+
+def dequantise_batch(planes, n: int, dtype=None, layout: str = "rows", outs=None, stream=None):
+    """``dequantise`` for several (codes, centres) planes of one vector length in one
+    launch (kd_dequantise_batch); returns one dense matrix per plane."""
+    torch = _torch()
+    if not 1 <= len(planes) <= KD_MAX_BATCH:
+        raise ValueError(f"1..{KD_MAX_BATCH} planes")
+    dtype = dtype or torch.float32
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    arr = (KdPlane * len(planes))()
+    res = []
+    for i, (codes, centres) in enumerate(planes):
+        m = codes.shape[0]
+        if outs is not None:
+            o = outs[i]
+        else:
+            o = torch.empty((m, n) if lay == KD_VEC_ROWS else (n, m), dtype=dtype, device=codes.device)
+        if o.dtype != dtype:
+            raise ValueError("outputs must share one dtype")
+        arr[i] = KdPlane(codes.data_ptr(), centres.data_ptr(), o.data_ptr(), m, o.stride(0))
+        res.append(o)
+    st = kd_dequantise_batch(ctypes.cast(arr, ctypes.c_void_p), len(planes), n, _dtype_code(dtype), lay,
+                             _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_dequantise_batch")
+    return res
 
 
 def rht(x, seed: int, inverse: bool = False, out=None, status=None, stream=None):

@@ -124,6 +124,17 @@ def test_argument_validation_without_gpu(kd):
     assert kd.kd_apply_p(null, 1, 256, 2, 0, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_reconstruct(1, 1, 1, 1, 256, 2, 0, 9, 0, 1, 256, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_read_status(null, null) == kd.KD_ERR_WORKSPACE
+    # batched dequantise: plane count and array
+    assert kd.kd_dequantise_batch(null, 1, 256, 0, 0, null) == kd.KD_ERR_INVALID_ARG
+    planes = (kd.KdPlane * 2)()
+    assert kd.kd_dequantise_batch(ctypes.cast(planes, ctypes.c_void_p), 0, 256, 0, 0, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_dequantise_batch(ctypes.cast(planes, ctypes.c_void_p), kd.KD_MAX_BATCH + 1, 256, 0, 0,
+                                  null) == kd.KD_ERR_INVALID_ARG
+    # a plane with m > 0 and null pointers, then one whose ld is too small
+    planes[0] = kd.KdPlane(None, None, None, 4, 256)
+    assert kd.kd_dequantise_batch(ctypes.cast(planes, ctypes.c_void_p), 1, 256, 0, 0, null) == kd.KD_ERR_INVALID_ARG
+    planes[0] = kd.KdPlane(16, 16, 16, 4, 255)
+    assert kd.kd_dequantise_batch(ctypes.cast(planes, ctypes.c_void_p), 1, 256, 0, 0, null) == kd.KD_ERR_INVALID_ARG
 
 
 def test_rht_block_and_validation(kd):

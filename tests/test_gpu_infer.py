@@ -67,6 +67,30 @@ def test_dequantise_ragged_length_and_strides(kd):
     assert bool((big[:, :3] == -7.0).all()) and bool((big[:, 103:] == -7.0).all())
 
 
+@pytest.mark.parametrize("n", [100, 4096])
+@pytest.mark.parametrize("layout", ["rows", "columns"])
+def test_dequantise_batch_equals_single_calls(kd, n, layout):
+    """One batched launch over planes of different vector counts (one of them empty,
+    one written into a strided view) writes every plane exactly as its own call."""
+    import torch
+    g = torch.Generator().manual_seed(n)
+    words = (n + 15) // 16
+    ms = [5, 0, 300, 1, 64]
+    planes = [(torch.randint(-2**31, 2**31 - 1, (m, words), generator=g, dtype=torch.int32).cuda(),
+               torch.sort(torch.randn((m, 4), generator=g), dim=1).values.cuda()) for m in ms]
+    for dtype in (torch.float32, torch.float16, torch.bfloat16):
+        outs = []
+        for (c, _), m in zip(planes, ms):
+            shape = (m, n + 24) if layout == "rows" else (n, m + 24)
+            outs.append(torch.full(shape, -3.0, dtype=dtype, device="cuda")[:, 8:(n if layout == "rows" else m) + 8])
+        got = kd.dequantise_batch(planes, n, dtype=dtype, layout=layout, outs=outs)
+        for (c, cent), o in zip(planes, got):
+            one = kd.dequantise(c, cent, n, dtype=dtype, layout=layout)
+            torch.cuda.synchronize()
+            assert torch.equal(o, one)
+            assert bool((o._base[:, :8] == -3.0).all()) and bool((o._base[:, -16:] == -3.0).all())
+
+
 @pytest.mark.parametrize("n,m,t", [(768, 33, 5), (4096, 12, 8), (11008, 6, 3)])
 def test_folding_identity(kd, n, m, t):
     """App. C: X W_hat computed three ways -- dense W_hat from kd_reconstruct, the
