@@ -95,8 +95,8 @@ kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host);
  * factors (Sec. 3.2 Algorithm 1; Sec. 2.1; App. C storage format).
  *
  *  w          input, dtype elements, `layout` with leading dimension ld.
- *  iters      k >= 0 blocks of four atomic greedy steps (two on Q_N -> u, two on
- *             P Q_N -> vhat).  k = 0 gives zero factors, zero centres, codes 0.
+ *  iters      k blocks (0 <= k <= 65536) of four atomic greedy steps (two on Q_N -> u,
+ *             two on P Q_N -> vhat).  k = 0 gives zero factors, zero centres, codes 0.
  *  kmeans_iters  0..64 Lloyd refinement iterations of each factor's 4 centres from
  *             the closed form (Sec. 2.1 refines the closed-form centres with a few
  *             k-means iterations): every entry goes to its nearest centre (ties to the
@@ -118,6 +118,11 @@ kd_status kd_signs(uint64_t sign_seed, int64_t n, int8_t* eps_host);
  *             does not change any other output bit.
  *  workspace  device scratch, 16-byte aligned (as cudaMalloc returns), of
  *             ws_bytes >= kd_workspace_size(n).
+ *
+ * Errors (returned before anything is enqueued): KD_ERR_INVALID_ARG for a bad size,
+ * count or enum, ld too small, a null required pointer with m > 0, or a pointer not
+ * aligned to its element (w to its dtype, codes and fp32 outputs to 4 bytes);
+ * KD_ERR_UNSUPPORTED_N; KD_ERR_WORKSPACE.  KD_ERR_CUDA if a launch fails.
  *
  * Vectors are processed two at a time (2j, 2j+1); each vector's results depend
  * only on its own data and its pair partner's (through rounding only). */
@@ -185,14 +190,16 @@ kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, k
 
 /* y_j = P x_j for m vectors of length n, fp32, vector-major [m][n] contiguous
  * (Sec. 3.1: P z = IDCT(eps * DCT(z)); App. C uses the same operator on the rows
- * of the activations, XP).  x and y may alias. */
+ * of the activations, XP).  x and y may alias; both 4-byte aligned
+ * (KD_ERR_INVALID_ARG otherwise). */
 kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t sign_seed,
                      void* workspace, size_t ws_bytes, void* stream);
 
 /* Dense re-materialisation W_hat = U_q + P V_q (App. C): vector j of w_hat is
  * centres_u[j][code_u] + P(centres_v[j][code_v]).  Inputs as produced by
- * kd_decompose (centres 16-byte aligned, KD_ERR_INVALID_ARG otherwise); output dtype
- * out_dtype in `layout` with leading dimension ld. */
+ * kd_decompose (centres 16-byte aligned, codes 4-byte aligned, KD_ERR_INVALID_ARG
+ * otherwise); output dtype out_dtype in `layout` with leading dimension ld, aligned
+ * to its element. */
 kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v,
                          const float* centres_u, const float* centres_v, int64_t n, int64_t m,
                          uint64_t sign_seed, kd_dtype out_dtype, kd_layout layout, void* w_hat,

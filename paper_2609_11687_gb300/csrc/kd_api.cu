@@ -119,6 +119,21 @@ int grid_for(int64_t npairs, int q, int ctas_max) {
 }
 
 bool valid_dtype(int d) { return d == KD_F32 || d == KD_F16 || d == KD_BF16; }
+
+// Blocks k and refinement iterations a call may ask for (keeps every step and trace
+// row count far inside int range).
+constexpr int kMaxIters = 1 << 16;
+
+// Every pointer a decomposition reads or writes element-wise must be aligned to its
+// element: the input to its dtype, the code words and fp32 outputs to 4 bytes.
+bool aligned_to(const void* ptr, size_t a) { return reinterpret_cast<uintptr_t>(ptr) % a == 0; }
+bool outputs_aligned(const void* w, int dtype, const void* codes_u, const void* codes_v, const void* centres_u,
+                     const void* centres_v, const void* coeffs, const void* u, const void* vhat, const void* resid) {
+  const size_t esz = dtype == KD_F32 ? 4 : 2;
+  return aligned_to(w, esz) && aligned_to(codes_u, 4) && aligned_to(codes_v, 4) && aligned_to(centres_u, 4) &&
+         aligned_to(centres_v, 4) && aligned_to(coeffs, 4) && aligned_to(u, 4) && aligned_to(vhat, 4) &&
+         aligned_to(resid, 4);
+}
 bool valid_layout(int l) { return l == KD_VEC_ROWS || l == KD_VEC_COLUMNS; }
 
 }  // namespace
@@ -170,13 +185,15 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
                        uint64_t sign_seed, int iters, int kmeans_iters, uint32_t* codes_u, uint32_t* codes_v,
                        float* centres_u, float* centres_v, float* coeffs, float* u, float* vhat,
                        float* resid, int8_t* trace, void* workspace, size_t ws_bytes, void* stream) {
-  if (n <= 0 || m < 0 || iters < 0 || kmeans_iters < 0 || kmeans_iters > 64 || !valid_dtype(dtype) ||
-      !valid_layout(layout))
+  if (n <= 0 || m < 0 || iters < 0 || iters > kMaxIters || kmeans_iters < 0 || kmeans_iters > 64 ||
+      !valid_dtype(dtype) || !valid_layout(layout))
     return KD_ERR_INVALID_ARG;
   const PlanOps* ops = plan_ops(n);
   if (!ops) return KD_ERR_UNSUPPORTED_N;
   if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
   if (m > 0 && (!w || !codes_u || !codes_v || !centres_u || !centres_v)) return KD_ERR_INVALID_ARG;
+  if (!outputs_aligned(w, dtype, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat, resid))
+    return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
   if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
@@ -224,8 +241,8 @@ size_t kd_workspace_size_batch(int64_t n, int count) {
 kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, kd_layout layout, int64_t n,
                              int iters, int kmeans_iters, void* workspace, size_t ws_bytes, void* stream) {
   static_assert(KD_MAX_BATCH == kMaxBatch, "batch limit of the header and the kernel");
-  if (!mats || count < 1 || count > KD_MAX_BATCH || n <= 0 || iters < 0 || kmeans_iters < 0 ||
-      kmeans_iters > 64 || !valid_dtype(dtype) || !valid_layout(layout))
+  if (!mats || count < 1 || count > KD_MAX_BATCH || n <= 0 || iters < 0 || iters > kMaxIters ||
+      kmeans_iters < 0 || kmeans_iters > 64 || !valid_dtype(dtype) || !valid_layout(layout))
     return KD_ERR_INVALID_ARG;
   const PlanOps* ops = plan_ops(n);
   if (!ops) return KD_ERR_UNSUPPORTED_N;
@@ -236,6 +253,9 @@ kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, k
     const kd_matrix& a = mats[i];
     if (a.m < 0 || (layout == KD_VEC_ROWS ? a.ld < n : a.ld < a.m)) return KD_ERR_INVALID_ARG;
     if (a.m > 0 && (!a.w || !a.codes_u || !a.codes_v || !a.centres_u || !a.centres_v)) return KD_ERR_INVALID_ARG;
+    if (!outputs_aligned(a.w, dtype, a.codes_u, a.codes_v, a.centres_u, a.centres_v, a.coeffs, nullptr, nullptr,
+                         nullptr))
+      return KD_ERR_INVALID_ARG;
     BatchMat& b = bp.mat[i];
     b.w = a.w;
     b.m = a.m;
@@ -304,6 +324,7 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
   const PlanOps* ops = plan_ops(n);
   if (!ops) return KD_ERR_UNSUPPORTED_N;
   if (m > 0 && (!x || !y)) return KD_ERR_INVALID_ARG;
+  if (!aligned_to(x, 4) || !aligned_to(y, 4)) return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
   if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
@@ -336,6 +357,8 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
   if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
   if (m > 0 && (!codes_u || !codes_v || !centres_u || !centres_v || !w_hat)) return KD_ERR_INVALID_ARG;
   if (m > 0 && ((reinterpret_cast<uintptr_t>(centres_u) | reinterpret_cast<uintptr_t>(centres_v)) % 16 != 0))
+    return KD_ERR_INVALID_ARG;
+  if (!aligned_to(codes_u, 4) || !aligned_to(codes_v, 4) || !aligned_to(w_hat, out_dtype == KD_F32 ? 4 : 2))
     return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;

@@ -112,15 +112,26 @@ def test_argument_validation_without_gpu(kd):
     # missing required outputs
     assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, null, 1, 1, 1, null, null, null, null, null, 1, 1 << 20,
                            null) == kd.KD_ERR_INVALID_ARG
+    # more blocks than the library accepts
+    assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, (1 << 16) + 1, 0, 16, 16, 16, 16, null, null, null, null, null,
+                           16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    # input or outputs not aligned to their elements
+    assert kd.kd_decompose(2, 0, 0, 256, 4, 256, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null, 16, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, 4, 0, 16, 18, 16, 16, null, null, null, null, null, 16, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, 4, 0, 16, 16, 16, 16, null, 6, null, null, null, 16, 1 << 20,
+                           null) == kd.KD_ERR_INVALID_ARG
     # workspace missing / too small
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, null, 1 << 20,
+    assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null, null, 1 << 20,
                            null) == kd.KD_ERR_WORKSPACE
-    assert kd.kd_decompose(1, 0, 0, 256, 4, 256, 0, 4, 0, 1, 1, 1, 1, null, null, null, null, null, 1, 16,
+    assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null, 16, 16,
                            null) == kd.KD_ERR_WORKSPACE
     # workspace not 16-byte aligned (its tables are read with 128-bit loads)
     assert kd.kd_decompose(16, 0, 0, 256, 4, 256, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null, 8, 1 << 20,
                            null) == kd.KD_ERR_WORKSPACE
-    assert kd.kd_apply_p(1, 1, 256, 2, 0, null, 0, null) == kd.KD_ERR_WORKSPACE
+    assert kd.kd_apply_p(16, 16, 256, 2, 0, null, 0, null) == kd.KD_ERR_WORKSPACE
+    assert kd.kd_apply_p(16, 6, 256, 2, 0, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG   # y not 4-byte aligned
     assert kd.kd_apply_p(null, 1, 256, 2, 0, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_reconstruct(1, 1, 1, 1, 256, 2, 0, 9, 0, 1, 256, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_read_status(null, null) == kd.KD_ERR_WORKSPACE
