@@ -463,9 +463,6 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
     fp16 out; one P per vector pair, ALU-bound) and the two expanded factor planes
     for the folded product [X | XP][U_q; V_q] (kd_dequantise, fp16 out, HBM-bound)."""
     decs = [(s, kd.decompose(w, iters, s.sign_seed, workspace=wss[s.N], stream=stream)) for s, w in layer]
-    outs = {}
-    for s, _ in layer:
-        outs.setdefault((s.M, s.N), torch.empty((s.M, s.N), dtype=torch.float16, device=layer[0][1].device))
     # both factor planes of every matrix, grouped by vector length: one batched launch each
     groups = {}
     for s, d in decs:
@@ -485,10 +482,17 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
         torch.cuda.synchronize()
         return sum(a.elapsed_time(b) for a, b in evs) / len(evs)
 
+    # every matrix to its own output, the matrices of one vector length in one launch
+    rec_groups = {}
+    for s, d in decs:
+        rec_groups.setdefault(s.N, []).append((s, d, torch.empty((s.M, s.N), dtype=torch.float16,
+                                                                 device=layer[0][1].device)))
+    wsr = {n: kd.Workspace(n, layer[0][1].device, count=len(g)) for n, g in rec_groups.items()}
+
     def rec():
-        for s, d in decs:
-            kd.reconstruct(d, s.N, s.sign_seed, dtype=torch.float16, out=outs[(s.M, s.N)],
-                           workspace=wss[s.N], stream=stream)
+        for n, grp in rec_groups.items():
+            kd.reconstruct_batch([d for _, d, _ in grp], n, [s.sign_seed for s, _, _ in grp], dtype=torch.float16,
+                                 outs=[o for _, _, o in grp], workspace=wsr[n], stream=stream)
 
     def deq():
         for n, pl in groups.items():
@@ -503,9 +507,10 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
     peak_alu = SM_COUNT * FP32_LANES_PER_SM * 2 * 2.070e9 / 1e12
     deq_bytes = 2 * params * (0.25 + 2)
     hbm, basis = hbm_peak_gbs()
-    del outs, decs, planes_out
+    del decs, planes_out, rec_groups
     return {
-        "reconstruct": {"kernel": "reconstruct_kernel (codes -> fp16 W_hat, 7 launches per layer)",
+        "reconstruct": {"kernel": "reconstruct_kernel (codes -> fp16 W_hat, one kd_reconstruct_batch per vector "
+                                  "length)",
                         "ms_per_layer": round(ms_rec, 4), "params_per_s": round(params / (ms_rec / 1e3), 1),
                         "bound": "alu", "achieved": round(flops / (ms_rec / 1e3) / 1e12, 3),
                         "peak": round(peak_alu, 2), "unit": "TFLOP/s",
@@ -524,9 +529,9 @@ def measure_rht(kd, torch, layer, stream):
     preprocessing): fp16 in, fp32 out, one kd_rht per matrix, timed with events on
     the launch stream.  HBM-bound: 2 B read + 4 B written per parameter.  Reported
     per layer (seven launches back to back) and per launch (the largest matrix)."""
-    outs = {}
-    for s, w in layer:
-        outs.setdefault(tuple(w.shape), torch.empty(tuple(w.shape), dtype=torch.float32, device=w.device))
+    # every matrix to its own output (outputs shared by equal shapes would let L2 absorb
+    # part of the writes)
+    outs = [torch.empty(tuple(w.shape), dtype=torch.float32, device=w.device) for _, w in layer]
     evs, big = [], []
     biggest = max(range(len(layer)), key=lambda i: layer[i][0].params)
     for rep in range(4):
@@ -538,7 +543,7 @@ def measure_rht(kd, torch, layer, stream):
                 c = torch.cuda.Event(enable_timing=True)
                 d = torch.cuda.Event(enable_timing=True)
                 c.record(stream)
-            kd.rht(w, RHT_SEED, out=outs[tuple(w.shape)], stream=stream)
+            kd.rht(w, RHT_SEED, out=outs[i], stream=stream)
             if i == biggest:
                 d.record(stream)
                 if rep > 0:

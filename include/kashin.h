@@ -205,6 +205,31 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v,
                          uint64_t sign_seed, kd_dtype out_dtype, kd_layout layout, void* w_hat,
                          int64_t ld, void* workspace, size_t ws_bytes, void* stream);
 
+/* kd_reconstruct for several matrices of one vector length n in one launch (App. C
+ * at load time: a layer's matrices together), each with its own codes, centres, sign
+ * seed, output and ld; out_dtype and layout are shared.  Every matrix is written
+ * exactly as kd_reconstruct would write it.
+ *   mats       HOST array of `count` descriptors (1 <= count <= KD_MAX_BATCH), read
+ *              during the call.
+ *   workspace  16-byte aligned, ws_bytes >= kd_workspace_size_batch(n, count) (one
+ *              sign set per matrix).
+ * Lengths above 8192 run one launch per matrix, in order, on the same stream and
+ * workspace.  Errors as kd_reconstruct (the first invalid matrix's), and
+ * KD_ERR_INVALID_ARG for a bad count or a null array. */
+typedef struct kd_recmat {
+  const uint32_t* codes_u;
+  const uint32_t* codes_v;
+  const float* centres_u;
+  const float* centres_v;
+  uint64_t sign_seed;
+  void* w_hat;
+  int64_t m;
+  int64_t ld;
+} kd_recmat;
+
+kd_status kd_reconstruct_batch(const kd_recmat* mats, int count, int64_t n, kd_dtype out_dtype, kd_layout layout,
+                               void* workspace, size_t ws_bytes, void* stream);
+
 /* Synchronises `stream` and returns KD_ERR_NONFINITE if any vector decomposed
  * by the last kd_decompose on this workspace held a NaN or Inf, KD_OK otherwise
  * (KD_ERR_CUDA if the synchronisation fails). */

@@ -113,6 +113,23 @@ kd_status setup(const PlanOps* ops, const WsLayout& L, void* ws, uint64_t seed, 
   return e == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
+// Tables of a batched call: twiddles, status and sign set 0 from the first seed, then
+// sign sets 1 .. count-1 (set i at eps + i * ceil(n / 32)).
+kd_status setup_batch(const PlanOps* ops, const WsLayout& L, void* ws, const uint64_t* seeds, int count, int64_t n,
+                      cudaStream_t s) {
+  kd_status st = setup(ops, L, ws, seeds[0], s);
+  if (st != KD_OK || count == 1) return st;
+  SeedList sl;
+  sl.count = count;
+  sl.words = (int)((n + 31) / 32);
+  sl.n = n;
+  for (int i = 0; i < count; ++i) sl.seed[i] = seeds[i];
+  const int total = count * sl.words;
+  eps_batch_kernel<<<(total + 255) / 256, 256, 0, s>>>(reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + L.eps),
+                                                       sl);
+  return cudaGetLastError() == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
 int grid_for(int64_t npairs, int q, int ctas_max) {
   const int64_t want = (npairs + q - 1) / q;
   return (int)(want < ctas_max ? want : ctas_max);
@@ -283,19 +300,11 @@ kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, k
     }
     return KD_OK;
   }
-  kd_status st = setup(ops, L, workspace, mats[0].sign_seed, s);  // twiddles, status, set 0
+  uint64_t seeds[KD_MAX_BATCH];
+  for (int i = 0; i < count; ++i) seeds[i] = mats[i].sign_seed;
+  kd_status st = setup_batch(ops, L, workspace, seeds, count, n, s);
   if (st != KD_OK) return st;
   char* b = static_cast<char*>(workspace);
-  SeedList sl;
-  sl.count = count;
-  sl.words = (int)((n + 31) / 32);
-  sl.n = n;
-  for (int i = 0; i < count; ++i) sl.seed[i] = mats[i].sign_seed;
-  if (count > 1) {  // set 0 came with the twiddles
-    const int total = count * sl.words;
-    eps_batch_kernel<<<(total + 255) / 256, 256, 0, s>>>(reinterpret_cast<uint32_t*>(b + L.eps), sl);
-    if (cudaGetLastError() != cudaSuccess) return KD_ERR_CUDA;
-  }
   if (npairs == 0) return KD_OK;
   DecParams p;
   std::memset(&p, 0, sizeof(p));
@@ -385,7 +394,70 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, per * sms);
-  return ops->reconstruct(p, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+  return ops->reconstruct(p, nullptr, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+kd_status kd_reconstruct_batch(const kd_recmat* mats, int count, int64_t n, kd_dtype out_dtype, kd_layout layout,
+                               void* workspace, size_t ws_bytes, void* stream) {
+  if (!mats || count < 1 || count > KD_MAX_BATCH || n <= 0 || !valid_dtype(out_dtype) || !valid_layout(layout))
+    return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  RecBatch rb;
+  rb.count = count;
+  int64_t npairs = 0;
+  for (int i = 0; i < count; ++i) {
+    const kd_recmat& a = mats[i];
+    if (a.m < 0 || (layout == KD_VEC_ROWS ? a.ld < n : a.ld < a.m)) return KD_ERR_INVALID_ARG;
+    if (a.m > 0 && (!a.codes_u || !a.codes_v || !a.centres_u || !a.centres_v || !a.w_hat)) return KD_ERR_INVALID_ARG;
+    if (!aligned_to(a.centres_u, 16) || !aligned_to(a.centres_v, 16) || !aligned_to(a.codes_u, 4) ||
+        !aligned_to(a.codes_v, 4) || !aligned_to(a.w_hat, out_dtype == KD_F32 ? 4 : 2))
+      return KD_ERR_INVALID_ARG;
+    RecMat& r = rb.mat[i];
+    r.codes_u = a.codes_u;
+    r.codes_v = a.codes_v;
+    r.centres_u = a.centres_u;
+    r.centres_v = a.centres_v;
+    r.out = a.w_hat;
+    r.m = a.m;
+    r.ld = a.ld;
+    r.pair0 = npairs;
+    npairs += (a.m + 1) / 2;
+  }
+  WsLayout L;
+  if (!layout_of(ops, &L, count)) return KD_ERR_CUDA;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!ops->batch) {
+    // long vectors: one launch per matrix on the same workspace, in stream order
+    for (int i = 0; i < count; ++i) {
+      const kd_recmat& a = mats[i];
+      const kd_status sti = kd_reconstruct(a.codes_u, a.codes_v, a.centres_u, a.centres_v, n, a.m, a.sign_seed,
+                                           out_dtype, layout, a.w_hat, a.ld, workspace, ws_bytes, stream);
+      if (sti != KD_OK) return sti;
+    }
+    return KD_OK;
+  }
+  uint64_t seeds[KD_MAX_BATCH];
+  for (int i = 0; i < count; ++i) seeds[i] = mats[i].sign_seed;
+  kd_status st = setup_batch(ops, L, workspace, seeds, count, n, s);
+  if (st != KD_OK || npairs == 0) return st;
+  char* b = static_cast<char*>(workspace);
+  RecParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.dtype = (int)out_dtype;
+  p.layout = (int)layout;
+  p.n = n;
+  p.m = mats[0].m;
+  p.ld = mats[0].ld;
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.npairs = npairs;
+  const int per = ops->ctas_per_sm(2, n);
+  const int sms = sm_count();
+  if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
+  const int grid = grid_for(p.npairs, ops->q, per * sms);
+  return ops->reconstruct(p, &rb, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
 kd_status kd_read_status(const void* workspace, void* stream) {

@@ -628,9 +628,9 @@ cudaError_t gen_apply_launch(const ApplyParams& p, int grid, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t gen_reconstruct(const RecParams& p, int grid, cudaStream_t s) {
+cudaError_t gen_reconstruct(const RecParams& p, const RecBatch* rb, int grid, cudaStream_t s) {
   GenPlan g;
-  if (!gen_plan(p.n, &g)) return cudaErrorInvalidValue;
+  if (rb || !gen_plan(p.n, &g)) return cudaErrorInvalidValue;
   const size_t smem = gen_smem(p.n);
   cudaError_t e = cudaFuncSetAttribute(gen_reconstruct_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;

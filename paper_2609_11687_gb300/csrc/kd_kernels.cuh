@@ -666,8 +666,24 @@ struct RecParams {
   int64_t npairs;
 };
 
+// Several matrices of one vector length in one reconstruct launch
+// (kd_reconstruct_batch): matrix i owns the global pairs [pair0, pair0 + ceil(m / 2))
+// and the sign bits at eps + i * ceil(n / 32); dtype and layout are shared.
+struct RecMat {
+  const uint32_t* codes_u;
+  const uint32_t* codes_v;
+  const float* centres_u;
+  const float* centres_v;
+  void* out;
+  int64_t m, ld, pair0;
+};
+struct RecBatch {
+  int count;  // 0: the single matrix of RecParams
+  RecMat mat[kMaxBatch];
+};
+
 template <class PL>
-__global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecParams p) {
+__global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecParams p, const __grid_constant__ RecBatch rb) {
   constexpr int N = PL::N;
   constexpr int T = PL::T;
   constexpr int E = PL::E;
@@ -679,18 +695,36 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
   float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
   Xform<PL> xf;
   xf.init(buf, tw, p.eps, lt);
+  int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
     const bool active = pair < p.npairs;
-    const int64_t pr = active ? pair : base;
+    int64_t pr = active ? pair : base;
+    // this pair's matrix: index mi into rb (batched launch) or RecParams' matrix; its
+    // fields are re-read from the parameter space where used
+    int mi = 0;
+    const bool batched = PL::BATCH && rb.count > 0;
+    if (batched) {
+      while (mi + 1 < rb.count && pr >= rb.mat[mi + 1].pair0) ++mi;
+      pr -= rb.mat[mi].pair0;
+      if (mi != cur_mat) {  // uniform per team: Q == 1 whenever T > 32
+        xf.set_eps(p.eps + (int64_t)mi * ((N + 31) / 32));
+        cur_mat = mi;
+      }
+    }
+    const uint32_t* codes_u = batched ? rb.mat[mi].codes_u : p.codes_u;
+    const uint32_t* codes_v = batched ? rb.mat[mi].codes_v : p.codes_v;
+    const float* centres_u = batched ? rb.mat[mi].centres_u : p.centres_u;
+    const float* centres_v = batched ? rb.mat[mi].centres_v : p.centres_v;
+    const int64_t m_in = batched ? rb.mat[mi].m : p.m;
     const int64_t colA = 2 * pr;
-    const bool hasB = (colA + 1) < p.m;
+    const bool hasB = (colA + 1) < m_in;
     const int64_t colB = hasB ? colA + 1 : colA;
     // the four centre sets of the pair (the same for the whole team: broadcast loads)
-    const float4 cuA = __ldg(reinterpret_cast<const float4*>(p.centres_u) + colA);
-    const float4 cuB = __ldg(reinterpret_cast<const float4*>(p.centres_u) + colB);
-    const float4 cvA = __ldg(reinterpret_cast<const float4*>(p.centres_v) + colA);
-    const float4 cvB = __ldg(reinterpret_cast<const float4*>(p.centres_v) + colB);
+    const float4 cuA = __ldg(reinterpret_cast<const float4*>(centres_u) + colA);
+    const float4 cuB = __ldg(reinterpret_cast<const float4*>(centres_u) + colB);
+    const float4 cvA = __ldg(reinterpret_cast<const float4*>(centres_v) + colA);
+    const float4 cvB = __ldg(reinterpret_cast<const float4*>(centres_v) + colB);
     auto pick = [](const float4& c, uint32_t q) -> float {
       const float lo = (q & 1u) ? c.y : c.x;
       const float hi = (q & 1u) ? c.w : c.z;
@@ -699,8 +733,8 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
     // code words of the pair staged in shared memory, word w as (uA, uB, vA, vB)
     uint4* cw = reinterpret_cast<uint4*>(buf);
     for (int w = lt; w < WPV; w += T) {
-      cw[w] = make_uint4(__ldg(&p.codes_u[colA * WPV + w]), __ldg(&p.codes_u[colB * WPV + w]),
-                         __ldg(&p.codes_v[colA * WPV + w]), __ldg(&p.codes_v[colB * WPV + w]));
+      cw[w] = make_uint4(__ldg(&codes_u[colA * WPV + w]), __ldg(&codes_u[colB * WPV + w]),
+                         __ldg(&codes_v[colA * WPV + w]), __ldg(&codes_v[colB * WPV + w]));
     }
     team_sync<PL>();
     float2 uq[E], vq[E];
@@ -723,13 +757,15 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
     }
     team_sync<PL>();
     if (active) {
+      void* out = batched ? rb.mat[mi].out : p.out;
+      const int64_t ld = batched ? rb.mat[mi].ld : p.ld;
       for (int i = 2 * lt; i < N; i += 2 * T) {
         const float2 e0 = buf[i], e1 = buf[i + 1];   // entries i, i + 1 of (A, B)
-        store_elem(p.out, p.dtype, elem_index(p.layout, colA, i, p.ld), e0.x);
-        store_elem(p.out, p.dtype, elem_index(p.layout, colA, i + 1, p.ld), e1.x);
+        store_elem(out, p.dtype, elem_index(p.layout, colA, i, ld), e0.x);
+        store_elem(out, p.dtype, elem_index(p.layout, colA, i + 1, ld), e1.x);
         if (hasB) {
-          store_elem(p.out, p.dtype, elem_index(p.layout, colB, i, p.ld), e0.y);
-          store_elem(p.out, p.dtype, elem_index(p.layout, colB, i + 1, p.ld), e1.y);
+          store_elem(out, p.dtype, elem_index(p.layout, colB, i, ld), e0.y);
+          store_elem(out, p.dtype, elem_index(p.layout, colB, i + 1, ld), e1.y);
         }
       }
     }

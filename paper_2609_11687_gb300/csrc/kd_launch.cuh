@@ -36,11 +36,16 @@ struct Ops {
     }
     return cudaGetLastError();
   }
-  static cudaError_t reconstruct(const RecParams& p, int grid, cudaStream_t s) {
+  static cudaError_t reconstruct(const RecParams& p, const RecBatch* rb, int grid, cudaStream_t s) {
     auto k = reconstruct_kernel<PL>;
     cudaError_t e = prepare(k, PL::SMEM);
     if (e != cudaSuccess) return e;
-    k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
+    if (rb) {
+      k<<<grid, PL::THREADS, PL::SMEM, s>>>(p, *rb);
+    } else {
+      RecBatch none{};
+      k<<<grid, PL::THREADS, PL::SMEM, s>>>(p, none);
+    }
     return cudaGetLastError();
   }
   static cudaError_t apply(const ApplyParams& p, int grid, cudaStream_t s) {

@@ -11,6 +11,7 @@ struct DecParams;
 struct BatchParams;
 struct ApplyParams;
 struct RecParams;
+struct RecBatch;
 
 struct PlanOps {
   int n;
@@ -25,7 +26,8 @@ struct PlanOps {
   // bp: the matrices of a batched launch, or nullptr for DecParams' single matrix
   cudaError_t (*decompose)(const DecParams&, const BatchParams* bp, int grid, cudaStream_t);
   cudaError_t (*apply)(const ApplyParams&, int grid, cudaStream_t);
-  cudaError_t (*reconstruct)(const RecParams&, int grid, cudaStream_t);
+  // rb: the matrices of a batched launch, or nullptr for RecParams' single matrix
+  cudaError_t (*reconstruct)(const RecParams&, const RecBatch* rb, int grid, cudaStream_t);
   // tables for one call of vector length n: twiddles (float2[twn]), sign bits, cleared status word
   cudaError_t (*setup)(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, int64_t n, cudaStream_t);
 };

@@ -32,13 +32,20 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
-           "kd_workspace_size_batch", "kd_decompose_batch")
+           "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
 
 
 class KdPlane(ctypes.Structure):
     """kd_plane: one 2-bit code plane to expand (kd_dequantise_batch)."""
     _fields_ = [("codes", ctypes.c_void_p), ("centres", ctypes.c_void_p), ("out", ctypes.c_void_p),
+                ("m", ctypes.c_int64), ("ld", ctypes.c_int64)]
+
+
+class KdRecMat(ctypes.Structure):
+    """kd_recmat: one matrix to re-materialise (kd_reconstruct_batch)."""
+    _fields_ = [("codes_u", ctypes.c_void_p), ("codes_v", ctypes.c_void_p), ("centres_u", ctypes.c_void_p),
+                ("centres_v", ctypes.c_void_p), ("sign_seed", ctypes.c_uint64), ("w_hat", ctypes.c_void_p),
                 ("m", ctypes.c_int64), ("ld", ctypes.c_int64)]
 
 
@@ -81,6 +88,8 @@ def _load() -> ctypes.CDLL:
     lib.kd_workspace_size_batch.restype = c_sz
     lib.kd_decompose_batch.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
     lib.kd_decompose_batch.restype = c_int
+    lib.kd_reconstruct_batch.argtypes = [c_vp, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
+    lib.kd_reconstruct_batch.restype = c_int
     lib.kd_measure_fp32_peak.argtypes = [c_vp, c_vp]
     lib.kd_measure_fp32_peak.restype = c_int
     lib.kd_dequantise.argtypes = [c_vp, c_vp, c_i64, c_i64, c_int, c_int, c_vp, c_i64, c_vp]
@@ -167,6 +176,10 @@ def kd_workspace_size_batch(n: int, count: int) -> int:
 
 def kd_decompose_batch(mats, count, dtype, layout, n, iters, kmeans_iters, workspace, ws_bytes, stream) -> int:
     return lib.kd_decompose_batch(mats, count, dtype, layout, n, iters, kmeans_iters, workspace, ws_bytes, stream)
+
+
+def kd_reconstruct_batch(mats, count, n, out_dtype, layout, workspace, ws_bytes, stream) -> int:
+    return lib.kd_reconstruct_batch(mats, count, n, out_dtype, layout, workspace, ws_bytes, stream)
 
 
 def kd_read_status(workspace, stream) -> int:
@@ -438,6 +451,35 @@ def reconstruct(dec: Decomposed, n: int, sign_seed: int, dtype=None, layout: str
     if st != KD_OK:
         raise KashinError(st, "kd_reconstruct")
     return out
+
+
+def reconstruct_batch(decs, n: int, sign_seeds, dtype=None, layout: str = "rows", outs=None,
+                      workspace: Optional[Workspace] = None, stream=None):
+    """``reconstruct`` for several decomposed matrices of one vector length in one
+    launch (kd_reconstruct_batch); returns one dense W_hat per matrix."""
+    torch = _torch()
+    if not 1 <= len(decs) <= KD_MAX_BATCH or len(sign_seeds) != len(decs):
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices with one seed each")
+    dtype = dtype or torch.float32
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    dev = decs[0].codes_u.device
+    arr = (KdRecMat * len(decs))()
+    res = []
+    for i, d in enumerate(decs):
+        m = d.codes_u.shape[0]
+        o = outs[i] if outs is not None else torch.empty((m, n) if lay == KD_VEC_ROWS else (n, m), dtype=dtype,
+                                                         device=dev)
+        if o.dtype != dtype:
+            raise ValueError("outputs must share one dtype")
+        arr[i] = KdRecMat(d.codes_u.data_ptr(), d.codes_v.data_ptr(), d.centres_u.data_ptr(), d.centres_v.data_ptr(),
+                          int(sign_seeds[i]) & ((1 << 64) - 1), o.data_ptr(), m, o.stride(0))
+        res.append(o)
+    ws = workspace if workspace is not None else Workspace(n, dev, count=len(decs))
+    st = kd_reconstruct_batch(ctypes.cast(arr, ctypes.c_void_p), len(decs), n, _dtype_code(dtype), lay, ws.ptr,
+                              ws.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_reconstruct_batch")
+    return res
 
 
 def unpack_codes(words, n: int):

@@ -135,6 +135,17 @@ def test_argument_validation_without_gpu(kd):
     assert kd.kd_apply_p(null, 1, 256, 2, 0, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_reconstruct(1, 1, 1, 1, 256, 2, 0, 9, 0, 1, 256, 1, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_read_status(null, null) == kd.KD_ERR_WORKSPACE
+    # batched reconstruct: matrix count and array
+    assert kd.kd_reconstruct_batch(null, 1, 256, 0, 0, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    recs = (kd.KdRecMat * 2)()
+    assert kd.kd_reconstruct_batch(ctypes.cast(recs, ctypes.c_void_p), 0, 256, 0, 0, 16, 1 << 20,
+                                   null) == kd.KD_ERR_INVALID_ARG
+    recs[0] = kd.KdRecMat(16, 16, 16, 16, 0, 16, 4, 256)
+    assert kd.kd_reconstruct_batch(ctypes.cast(recs, ctypes.c_void_p), 1, 4094, 0, 0, 16, 1 << 20,
+                                   null) == kd.KD_ERR_UNSUPPORTED_N
+    recs[0] = kd.KdRecMat(16, 16, 8, 16, 0, 16, 4, 256)   # centres not 16-byte aligned
+    assert kd.kd_reconstruct_batch(ctypes.cast(recs, ctypes.c_void_p), 1, 256, 0, 0, 16, 1 << 20,
+                                   null) == kd.KD_ERR_INVALID_ARG
     # batched dequantise: plane count and array
     assert kd.kd_dequantise_batch(null, 1, 256, 0, 0, null) == kd.KD_ERR_INVALID_ARG
     planes = (kd.KdPlane * 2)()

@@ -67,6 +67,32 @@ def test_dequantise_ragged_length_and_strides(kd):
     assert bool((big[:, :3] == -7.0).all()) and bool((big[:, 103:] == -7.0).all())
 
 
+@pytest.mark.parametrize("n", [768, 4096, 11008])
+def test_reconstruct_batch_equals_single_calls(kd, n):
+    """One batched launch over matrices with their own seeds and vector counts (odd,
+    one, none) writes every W_hat exactly as its own kd_reconstruct call; n = 11008
+    takes the one-launch-per-matrix path."""
+    import torch
+    g = torch.Generator().manual_seed(n + 3)
+    words = (n + 15) // 16
+    ms = [7, 1, 0, 40] if n < 11008 else [3, 0, 2]
+    seeds = [11 * i + n for i in range(len(ms))]
+    decs = []
+    for m in ms:
+        cu = torch.sort(torch.randn((m, 4), generator=g), dim=1).values.cuda()
+        cv = torch.sort(torch.randn((m, 4), generator=g), dim=1).values.cuda()
+        decs.append(kd.Decomposed(
+            codes_u=torch.randint(-2**31, 2**31 - 1, (m, words), generator=g, dtype=torch.int32).cuda(),
+            codes_v=torch.randint(-2**31, 2**31 - 1, (m, words), generator=g, dtype=torch.int32).cuda(),
+            centres_u=cu, centres_v=cv, coeffs=None, u=None, vhat=None, resid=None, trace=None))
+    for dtype, layout in ((torch.float32, "rows"), (torch.float16, "rows"), (torch.float32, "columns")):
+        got = kd.reconstruct_batch(decs, n, seeds, dtype=dtype, layout=layout)
+        for d, sd, o in zip(decs, seeds, got):
+            one = kd.reconstruct(d, n, sd, dtype=dtype, layout=layout)
+            torch.cuda.synchronize()
+            assert torch.equal(o, one), (n, dtype, layout)
+
+
 @pytest.mark.parametrize("n", [100, 4096])
 @pytest.mark.parametrize("layout", ["rows", "columns"])
 def test_dequantise_batch_equals_single_calls(kd, n, layout):
