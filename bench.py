@@ -179,10 +179,12 @@ class ClockSampler:
 _ORACLE_P = {}
 
 
-def oracle_baseline(specs, iters: int, budget_s: float = 12.0, kmeans_iters: int = 0) -> dict:
+def oracle_baseline(specs, iters: int, budget_s: float = 20.0, kmeans_iters: int = 0) -> dict:
     """Time the CPU oracle as it stands on a bounded sample of the layer and scale
     to params/s of the whole layer mix (time per parameter measured per vector
-    length, weighted by the layer's parameters at that length)."""
+    length, weighted by the layer's parameters at that length).  Per length the
+    sample doubles until one run takes half its share of the budget (or reaches 512
+    vectors); that run is the measurement."""
     import numpy as np
     from oracle import kashin_oracle as ko
     from paper_2609_11687_gb300 import synth
@@ -216,7 +218,7 @@ def oracle_baseline(specs, iters: int, budget_s: float = 12.0, kmeans_iters: int
                 code_u, code_v = ko.codes(d.u, cu), ko.codes(d.vhat, cv)
             ko.pack_codes(code_u), ko.pack_codes(code_v)
             dt = time.perf_counter() - t0
-            if dt > share / 4 or m >= 512:
+            if dt > share / 2 or m >= 512:
                 break
             m = min(512, m * 2)
         per_param[n] = dt / (m * n)
@@ -771,7 +773,7 @@ def main():
                     help="synthetic stand-in per step (default: one Llama-2-7B-shaped layer)")
     ap.add_argument("--skip-cpu", action="store_true")
     ap.add_argument("--skip-e2e", action="store_true")
-    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--cpu-budget", type=float, default=20.0)
     ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
     ap.add_argument("--profile-m", type=int, default=32768)
     ap.add_argument("--profile-matrix", type=int, default=0, help="layer matrix index (0 = q, 6 = down)")
