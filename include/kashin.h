@@ -297,7 +297,8 @@ kd_status kd_dequantise_batch(const kd_plane* planes, int count, int64_t n, kd_d
  *   stream   cudaStream_t as void*.
  * Errors: KD_ERR_UNSUPPORTED_N unless n % 16 == 0 and 16 <= n <= 65536;
  * KD_ERR_INVALID_ARG for m < 0, ld too small, bad dtype or flag, null pointers
- * with m > 0, or an in-place call that is not fp32 with equal strides;
+ * with m > 0, x, y or status not aligned to their elements, or an in-place call
+ * that is not fp32 with equal strides;
  * KD_ERR_CUDA if the launch fails.  m == 0 enqueues nothing.  No workspace.
  * To rotate along the other axis of a matrix (the output side of a two-sided
  * rotation) pass its transpose. */

@@ -625,6 +625,10 @@ extern "C" kd_status kd_rht(const void* x, kd_dtype dtype, int64_t n, int64_t m,
     return KD_ERR_INVALID_ARG;
   if (m == 0) return KD_OK;
   if (!x || !y) return KD_ERR_INVALID_ARG;
+  // elements are read and written at least one at a time: aligned to their size
+  if (reinterpret_cast<uintptr_t>(x) % (dtype == KD_F32 ? 4 : 2) != 0 || reinterpret_cast<uintptr_t>(y) % 4 != 0 ||
+      reinterpret_cast<uintptr_t>(status) % 4 != 0)
+    return KD_ERR_INVALID_ARG;
   // in place only over the same fp32 array with the same stride
   if (static_cast<const void*>(y) == x && (dtype != KD_F32 || ldx != ldy)) return KD_ERR_INVALID_ARG;
   const int log_b = kd::log2_block(n);

@@ -175,6 +175,11 @@ def test_rht_block_and_validation(kd):
     # in place only for fp32 with equal strides
     assert kd.kd_rht(4096, 1, 256, 4, 256, 0, 0, 4096, 256, null, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_rht(4096, 0, 256, 4, 256, 0, 0, 4096, 512, null, null) == kd.KD_ERR_INVALID_ARG
+    # pointers not aligned to their elements
+    assert kd.kd_rht(4098, 0, 256, 4, 256, 0, 0, 8192, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(4097, 1, 256, 4, 256, 0, 0, 8192, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(4096, 1, 256, 4, 256, 0, 0, 8194, 256, null, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_rht(4096, 1, 256, 4, 256, 0, 0, 8192, 256, 6, null) == kd.KD_ERR_INVALID_ARG
     # nothing to do: no launch, no device needed
     assert kd.kd_rht(null, 0, 256, 0, 256, 0, 0, null, 256, null, null) == kd.KD_OK
 
