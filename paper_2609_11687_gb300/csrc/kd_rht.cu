@@ -196,11 +196,24 @@ __device__ __forceinline__ void load16(const RhtParams& p, int64_t o, float2 (&v
 // data arrive already sign-flipped and scaled.  `after_first_barrier` runs once
 // per unit right after the first CTA barrier, when every thread has finished
 // reading what it loaded the unit from.
-template <int LOG_B, bool INV, class F>
+//
+// UNIT_BAR: the caller passes a CTA barrier at the start of every unit, after the
+// previous unit's last reads of buf.  Then the first exchange needs no barrier
+// before its writes, and with three or more passes the exchange between passes 0
+// and 1 stays inside a half-warp: pass 0's 16 contiguous entries of thread t and
+// pass 1's 16-strided group of thread t both lie in the 256-entry run t / 16, which
+// threads 16 (t / 16) .. +15 alone write and read (both paddings keep a run inside
+// its own slots).  That exchange, and the writes of pass 1 into the next one, then
+// need only warp barriers.
+template <int LOG_B, bool INV, bool UNIT_BAR = false, class F>
 __device__ __forceinline__ void transform_and_store(const RhtParams& p, float2 (&v)[8], float* buf, int t,
                                                     bool active, int64_t j, int64_t off, uint32_t run_bits,
                                                     F&& after_first_barrier) {
   constexpr int NPASS = (LOG_B + 3) / 4;
+  constexpr bool LOCAL = UNIT_BAR && NPASS >= 3;
+  // the step whose read barrier is the first CTA barrier (forward: the exchange 0 -> 1
+  // is warp-local, so the second step's)
+  constexpr int FIRST_CTA = (LOCAL && !INV) ? 2 : 1;
   if constexpr (NPASS == 1) {
     __syncthreads();
     after_first_barrier();
@@ -213,14 +226,26 @@ __device__ __forceinline__ void transform_and_store(const RhtParams& p, float2 (
       constexpr int X = K < KP ? K : KP;  // exchange between passes X and X + 1
       const int wbase = rpad<X>(rht_base<LOG_B, KP>(t));
       const int rbase = rpad<X>(rht_base<LOG_B, K>(t));
-      __syncthreads();  // the previous unit's reads of buf (and of the load's source) are done
-      if constexpr (KI == 1) after_first_barrier();
+      // before the writes: the previous reads of the slots written here are done
+      if constexpr (UNIT_BAR && KI == 1) {
+        // the unit barrier ordered them
+      } else if constexpr (LOCAL && KP == 1) {
+        __syncwarp();  // pass 1's slots were read by this half-warp alone
+      } else {
+        __syncthreads();
+      }
+      if constexpr (!UNIT_BAR && KI == 1) after_first_barrier();
       static_for<0, 8>([&](auto kk) {
         constexpr int Q = decltype(kk)::value;
         *slot<LOG_B, KP, X, 2 * Q>(buf, wbase) = v[Q].x;
         *slot<LOG_B, KP, X, 2 * Q + 1>(buf, wbase) = v[Q].y;
       });
-      __syncthreads();
+      if constexpr (LOCAL && X == 0) {
+        __syncwarp();
+      } else {
+        __syncthreads();
+      }
+      if constexpr (UNIT_BAR && KI == FIRST_CTA) after_first_barrier();
       static_for<0, 8>([&](auto kk) {
         constexpr int Q = decltype(kk)::value;
         v[Q] = make_float2(*slot<LOG_B, K, X, 2 * Q>(buf, rbase), *slot<LOG_B, K, X, 2 * Q + 1>(buf, rbase));
@@ -537,7 +562,7 @@ __global__ void __launch_bounds__(rht_threads(LOG_B), rht_min_blocks(LOG_B)) rht
       parity ^= 1u;
     }
     // after the first barrier every read of stage s_now is done: refill it
-    transform_and_store<LOG_B, INV>(p, v, buf, t, active, j, off, run_bits, [&] {
+    transform_and_store<LOG_B, INV, true>(p, v, buf, t, active, j, off, run_bits, [&] {
       if (tid == 0 && i + STAGES < n_iter) {
         fence_proxy_async_smem();
         issue(i + STAGES, s_now);
