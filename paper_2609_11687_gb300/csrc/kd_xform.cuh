@@ -252,6 +252,12 @@ struct Xform {
   // pass 1, the last pass and the inverse pass 1, so only the exchanges into and
   // out of pass 0 cross warps: two CTA barriers per P instead of four.
   static constexpr bool WL = NP == 3 && PL::PAIRED && E == 16 && PL::R(1) == 16 && PL::RL == 16 && T == 256;
+  // Slot-order plans of shape R0 x 16 x 16 (n = 11008): the 16 pass-1 groups and the
+  // 16 last-pass groups of a 256-slot block are taken by the same 16 consecutive
+  // threads (group g goes to thread g mod T in both passes), so the exchange between
+  // passes 1 and 2, forward and inverse, stays inside a half-warp.
+  static constexpr bool L12 = NP == 3 && !PL::PAIRED && PL::R(1) == 16 && PL::S(1) == 16 && PL::RL == 16 &&
+                              T % 16 == 0;
   int g1;                      // warp-local: this thread's pass-1 group
   int p0, p1;                  // slot-order M: partner slot constants
   int pb0;                     // pad(lt): base of the pass-0 slots lt + j T
@@ -515,14 +521,18 @@ struct Xform {
       });
     } else {
       static_for<1, NP>([&](auto ii) {
-        pass<decltype(ii)::value, -1>();
-        team_sync<PL>();
+        constexpr int I = decltype(ii)::value;
+        pass<I, -1>();
+        if constexpr (L12 && I == 1) __syncwarp();
+        else team_sync<PL>();
       });
       middle_slots(v);
       team_sync<PL>();
       static_for<1, NP>([&](auto ii) {
-        pass<NP - decltype(ii)::value, +1>();
-        team_sync<PL>();
+        constexpr int I = decltype(ii)::value;
+        pass<NP - I, +1>();
+        if constexpr (L12 && I == 1) __syncwarp();
+        else team_sync<PL>();
       });
     }
     inv0(v);
