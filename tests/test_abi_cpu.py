@@ -233,3 +233,18 @@ def test_product_path_requires_library(tmp_path, monkeypatch):
     mod = importlib.util.module_from_spec(spec)
     with pytest.raises(ImportError):
         spec.loader.exec_module(mod)
+
+
+def test_batch_wrappers_validate_counts_on_the_host(kd):
+    """The batched wrappers refuse an empty batch, more than KD_MAX_BATCH entries and
+    seed lists of the wrong length before they touch any device memory."""
+    with pytest.raises(ValueError):
+        kd.dequantise_batch([], 256)
+    with pytest.raises(ValueError):
+        kd.dequantise_batch([(None, None)] * (kd.KD_MAX_BATCH + 1), 256)
+    with pytest.raises(ValueError):
+        kd.reconstruct_batch([None, None], 256, [1])
+    with pytest.raises(ValueError):
+        kd.reconstruct_batch([None] * (kd.KD_MAX_BATCH + 1), 256, list(range(kd.KD_MAX_BATCH + 1)))
+    with pytest.raises(ValueError):
+        kd.decompose_batch([None, None], 4, [1])
