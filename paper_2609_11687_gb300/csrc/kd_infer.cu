@@ -9,11 +9,10 @@
 // Bound by HBM: per entry 1/4 byte of codes is read and 2 or 4 bytes are written.
 // Row layout: one warp per vector, consecutive lanes writing consecutive 16-byte
 // chunks (two per code word for 16-bit output, four for fp32), each lane with the
-// code loads of four chunks in flight.  Column
-// layout: consecutive threads take consecutive vectors of the same word, so every
-// store instruction of a warp writes consecutive addresses.  One launch serves one
-// plane (kd_dequantise) or up to KD_MAX_BATCH planes of one length
-// (kd_dequantise_batch).
+// code loads of four chunks in flight.  Column layout: consecutive threads take
+// consecutive vectors of the same word, so every store instruction of a warp writes
+// consecutive addresses.  One launch serves one plane (kd_dequantise) or up to
+// KD_MAX_BATCH planes of one length (kd_dequantise_batch).
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -64,9 +63,10 @@ __device__ __forceinline__ void dequant_col_step(const DeqParams& p, int64_t b) 
 
 int64_t col_steps(const DeqParams& p) { return p.words * ((p.m + 255) / 256); }
 
-// Several planes of one vector length in one launch: plane i owns the CTA steps
-// [first[i], first[i + 1]) (its vectors in the row layout, its column steps in the
-// column layout); the grid strides over all of them.
+// Several planes of one vector length in one launch: plane i owns the work units
+// [first[i], first[i + 1]) (its vectors, one warp each, in the row layout; its
+// column steps, one CTA each, in the column layout); the grid strides over all of
+// them.
 struct DeqBatch {
   int count;
   int64_t first[KD_MAX_BATCH + 1];
