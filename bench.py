@@ -299,11 +299,12 @@ def run_gpu(args) -> dict:
     else:
         launches_per_step = 2 * len(layer0)
     ev_main = {}  # per-launch events of the dominant kernel
+    ev_other = {}  # per-launch events of the other vector lengths' kernels
 
     def run_layer(L, record=False):
         mats = layers[L]
         for n_, ix in groups.items():
-            rec = record and n_ == NDOM
+            rec = record
             if rec:
                 e0 = torch.cuda.Event(enable_timing=True)
                 e1 = torch.cuda.Event(enable_timing=True)
@@ -318,7 +319,8 @@ def run_gpu(args) -> dict:
                                  stream=stream, kmeans_iters=args.kmeans_iters)
             if rec:
                 e1.record(stream)
-                ev_main.setdefault("ev", []).append((e0, e1, sum(mats[i][0].M for i in ix)))
+                dst = ev_main.setdefault("ev", []) if n_ == NDOM else ev_other.setdefault(n_, [])
+                dst.append((e0, e1, sum(mats[i][0].M for i in ix)))
 
     for i in range(args.warmup):
         run_layer(my_layers[i])
@@ -391,6 +393,18 @@ def run_gpu(args) -> dict:
         roofline["frac_of_measured_fp32_peak"] = round(achieved_tflops / meas, 4)
     fl_fft = fft_flops_per_vector(NDOM, iters) * vec_per_launch
     roofline["achieved_fft_count"] = round(fl_fft / (dur / 1e3) / 1e12, 3)
+
+    def other_kernels():
+        out = []
+        for n_, evs in sorted(ev_other.items()):
+            d_ = sum(a.elapsed_time(b) for a, b, _ in evs) / len(evs)
+            v_ = sum(mm for _, _, mm in evs) / len(evs)
+            t_ = flops_per_vector(n_, iters) * v_ / (d_ / 1e3) / 1e12
+            out.append({"kernel": f"decompose_kernel<N={n_}>", "launch_ms": round(d_, 3),
+                        "achieved": round(t_, 3), "unit": "TFLOP/s", "frac": round(t_ / peak, 4)})
+        return out
+    if ev_other:
+        roofline["other_kernels"] = _extra(other_kernels)
 
     # k-means refinement (Sec. 2.1): cost of KM_PROBE Lloyd iterations on the dominant
     # kernel, timed on the same matrices right after the timed region
