@@ -138,21 +138,30 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
  * synchronisation).  The paper has no counterpart: this is a library convenience.
  * Same arguments and results as kd_decompose minus workspace/ws_bytes; the scratch
  * lives in a 160 KB static device array inside the library instead.
- *   - n <= 8192 whose workspace fits the array (the tuned lengths; the run-time-length
- *     path needs per-CTA slots that do not fit); otherwise KD_ERR_WORKSPACE and
- *     nothing is enqueued.
+ *   - Arguments are checked first, in kd_decompose's order and with its error codes;
+ *     then n must be at most 8192 and its tables must fit the array (the tuned
+ *     lengths; the run-time-length path needs per-CTA slots that do not fit),
+ *     otherwise KD_ERR_WORKSPACE.  Nothing is enqueued on any error.
  *   - Allocates nothing.  Every GPU that loads the library holds the array until exit.
  *   - All calls share the array (it keeps the last call's tables); each call rewrites
- *     what it needs on its own stream, so calls that overlap on the GPU race.
+ *     what it needs and clears the status word on its own stream, so calls that
+ *     overlap on the GPU race.
  *   - The first call on a device resolves the array's address (cudaGetSymbolAddress,
  *     once per device): make that first call before any stream capture.
- *   - Non-finite inputs still set the device status word, which lives in the static
- *     array and is not readable through this ABI. */
+ *   - A non-finite input sets the status word in the array; kd_read_status_static
+ *     reads it back. */
 kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
                               int64_t ld, uint64_t sign_seed, int iters, int kmeans_iters,
                               uint32_t* codes_u, uint32_t* codes_v, float* centres_u, float* centres_v,
                               float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
                               void* stream);
+
+/* kd_read_status for kd_decompose_static: synchronises `stream`, then returns
+ * KD_ERR_NONFINITE if a vector of the last kd_decompose_static call on the current
+ * device held a NaN or Inf, KD_OK otherwise (also when no static call ran yet), and
+ * KD_ERR_CUDA if a CUDA call fails.  Allocates nothing.  The word is shared like the
+ * rest of the array: a static call enqueued after the one of interest clears it. */
+kd_status kd_read_status_static(void* stream);
 
 /* ---------------------------------------------------------------------------
  * Several matrices of one vector length n in one launch (Algorithm 1 and the 2-bit
@@ -268,6 +277,11 @@ typedef struct kd_plane {
 kd_status kd_dequantise_batch(const kd_plane* planes, int count, int64_t n, kd_dtype out_dtype, kd_layout layout,
                               void* stream);
 
+/* Measured FP32 throughput of the current device in TFLOP/s (packed FFMA2 chains on
+ * every SM, best of three timed launches on `stream`; synchronises the stream).
+ * Used as the measured denominator of the transform kernels' ALU roofline. */
+kd_status kd_measure_fp32_peak(double* tflops, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:
  * the weights are rotated by a randomized Hadamard transform before the
@@ -302,11 +316,6 @@ kd_status kd_dequantise_batch(const kd_plane* planes, int count, int64_t n, kd_d
  * KD_ERR_CUDA if the launch fails.  m == 0 enqueues nothing.  No workspace.
  * To rotate along the other axis of a matrix (the output side of a two-sided
  * rotation) pass its transpose. */
-/* Measured FP32 throughput of the current device in TFLOP/s (packed FFMA2 chains on
- * every SM, best of three timed launches on `stream`; synchronises the stream).
- * Used as the measured denominator of the transform kernels' ALU roofline. */
-kd_status kd_measure_fp32_peak(double* tflops, void* stream);
-
 #define KD_RHT_ERR_TIMEOUT 1u
 int64_t kd_rht_block(int64_t n); /* block length b for vectors of length n, 0 if unsupported */
 kd_status kd_rht(const void* x, kd_dtype dtype, int64_t n, int64_t m, int64_t ldx, uint64_t seed, int inverse,

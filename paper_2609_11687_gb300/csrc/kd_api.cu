@@ -154,6 +154,21 @@ bool outputs_aligned(const void* w, int dtype, const void* codes_u, const void* 
 bool valid_layout(int l) { return l == KD_VEC_ROWS || l == KD_VEC_COLUMNS; }
 
 }  // namespace
+
+int check_decompose_args(const void* w, int dtype, int layout, int64_t n, int64_t m, int64_t ld, int iters,
+                         int kmeans_iters, const void* codes_u, const void* codes_v, const void* centres_u,
+                         const void* centres_v, const void* coeffs, const void* u, const void* vhat,
+                         const void* resid) {
+  if (n <= 0 || m < 0 || iters < 0 || iters > kMaxIters || kmeans_iters < 0 || kmeans_iters > 64 ||
+      !valid_dtype(dtype) || !valid_layout(layout))
+    return KD_ERR_INVALID_ARG;
+  if (!plan_ops(n)) return KD_ERR_UNSUPPORTED_N;
+  if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
+  if (m > 0 && (!w || !codes_u || !codes_v || !centres_u || !centres_v)) return KD_ERR_INVALID_ARG;
+  if (!outputs_aligned(w, dtype, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat, resid))
+    return KD_ERR_INVALID_ARG;
+  return KD_OK;
+}
 }  // namespace kd
 
 using namespace kd;
@@ -202,15 +217,10 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
                        uint64_t sign_seed, int iters, int kmeans_iters, uint32_t* codes_u, uint32_t* codes_v,
                        float* centres_u, float* centres_v, float* coeffs, float* u, float* vhat,
                        float* resid, int8_t* trace, void* workspace, size_t ws_bytes, void* stream) {
-  if (n <= 0 || m < 0 || iters < 0 || iters > kMaxIters || kmeans_iters < 0 || kmeans_iters > 64 ||
-      !valid_dtype(dtype) || !valid_layout(layout))
-    return KD_ERR_INVALID_ARG;
+  const kd_status chk = (kd_status)check_decompose_args(w, dtype, layout, n, m, ld, iters, kmeans_iters, codes_u, codes_v,
+                                             centres_u, centres_v, coeffs, u, vhat, resid);
+  if (chk != KD_OK) return chk;
   const PlanOps* ops = plan_ops(n);
-  if (!ops) return KD_ERR_UNSUPPORTED_N;
-  if (layout == KD_VEC_ROWS ? ld < n : ld < m) return KD_ERR_INVALID_ARG;
-  if (m > 0 && (!w || !codes_u || !codes_v || !centres_u || !centres_v)) return KD_ERR_INVALID_ARG;
-  if (!outputs_aligned(w, dtype, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat, resid))
-    return KD_ERR_INVALID_ARG;
   WsLayout L;
   if (!layout_of(ops, &L)) return KD_ERR_CUDA;
   if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;

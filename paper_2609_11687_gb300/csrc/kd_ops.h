@@ -32,6 +32,14 @@ struct PlanOps {
   cudaError_t (*setup)(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, int64_t n, cudaStream_t);
 };
 
+// Argument checks of kd_decompose, in its order and with its status codes (a kd_status
+// value): sizes, counts and enums, the plan for n, ld, required pointers, alignment.
+// The workspace is not checked here.
+int check_decompose_args(const void* w, int dtype, int layout, int64_t n, int64_t m, int64_t ld, int iters,
+                         int kmeans_iters, const void* codes_u, const void* codes_v, const void* centres_u,
+                         const void* centres_v, const void* coeffs, const void* u, const void* vhat,
+                         const void* resid);
+
 // The compiled plan of length n, else the run-time-length path (kd_generic.cu), else nullptr.
 const PlanOps* plan_ops(int64_t n);
 // The compiled plan of length n, or nullptr.

@@ -9,8 +9,9 @@
 // of a caller workspace, so it allocates nothing.
 //
 // Limits and sharing:
-//  - the array holds the tables of one vector length up to 8192;
-//    longer vectors are rejected with KD_ERR_WORKSPACE before anything is enqueued;
+//  - the array holds the tables of one vector length up to 8192; after the same
+//    argument checks as kd_decompose, longer vectors (and lengths whose tables do
+//    not fit) are rejected with KD_ERR_WORKSPACE before anything is enqueued;
 //  - every GPU that loads the library holds the array until the process exits;
 //  - all calls share it and it keeps the last call's contents; each call rewrites
 //    the tables and clears the status word on its own stream before its kernel
@@ -18,7 +19,9 @@
 //    enqueued on another stream before the first finished) race;
 //  - the first call on a device resolves the array's device address with
 //    cudaGetSymbolAddress (once per device, with that device current); make that
-//    first call before any stream capture.
+//    first call before any stream capture;
+//  - a non-finite input sets the status word at the start of the array, which
+//    kd_read_status_static copies back (after synchronising the caller's stream).
 #include <mutex>
 
 #include "kashin.h"
@@ -61,17 +64,29 @@ cudaError_t scratch_on_current_device(void** out) {
 
 extern "C" kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, int64_t n, int64_t m,
                                          int64_t ld, uint64_t sign_seed, int iters, int kmeans_iters,
-                                         uint32_t* codes_u,
-                                         uint32_t* codes_v, float* centres_u, float* centres_v, float* coeffs,
-                                         float* u, float* vhat, float* resid, int8_t* trace, void* stream) {
+                                         uint32_t* codes_u, uint32_t* codes_v, float* centres_u, float* centres_v,
+                                         float* coeffs, float* u, float* vhat, float* resid, int8_t* trace,
+                                         void* stream) {
+  // the caller's arguments first, exactly as kd_decompose checks them
+  const kd_status chk = (kd_status)kd::check_decompose_args(w, dtype, layout, n, m, ld, iters, kmeans_iters, codes_u,
+                                                            codes_v, centres_u, centres_v, coeffs, u, vhat, resid);
+  if (chk != KD_OK) return chk;
+  // then the array's limits
   if (n > kd::kStaticMaxN) return KD_ERR_WORKSPACE;
-  if (kd_supported(n) != KD_OK) return KD_ERR_UNSUPPORTED_N;
   const size_t need = kd_workspace_size(n);
   if (need == 0) return KD_ERR_CUDA;
   if (need > kd::kStaticBytes) return KD_ERR_WORKSPACE;
+  // and only then the device address (loads the module on first use)
   void* scratch = nullptr;
   if (kd::scratch_on_current_device(&scratch) != cudaSuccess) return KD_ERR_CUDA;
   return kd_decompose(w, dtype, layout, n, m, ld, sign_seed, iters, kmeans_iters, codes_u, codes_v, centres_u,
-                      centres_v,
-                      coeffs, u, vhat, resid, trace, scratch, kd::kStaticBytes, stream);
+                      centres_v, coeffs, u, vhat, resid, trace, scratch, kd::kStaticBytes, stream);
+}
+
+// The status word sits at the start of the array (offset 0 of the workspace layout,
+// which kd_decompose's set-up clears before every kernel).
+extern "C" kd_status kd_read_status_static(void* stream) {
+  void* scratch = nullptr;
+  if (kd::scratch_on_current_device(&scratch) != cudaSuccess) return KD_ERR_CUDA;
+  return kd_read_status(scratch, stream);
 }

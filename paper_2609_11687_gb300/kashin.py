@@ -31,6 +31,7 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
+           "kd_read_status_static",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
@@ -84,6 +85,11 @@ def _load() -> ctypes.CDLL:
     lib.kd_reconstruct.restype = c_int
     lib.kd_read_status.argtypes = [c_vp, c_vp]
     lib.kd_read_status.restype = c_int
+    lib.kd_decompose_static.argtypes = [c_vp, c_int, c_int, c_i64, c_i64, c_i64, c_u64, c_int, c_int,
+                                        c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]
+    lib.kd_decompose_static.restype = c_int
+    lib.kd_read_status_static.argtypes = [c_vp]
+    lib.kd_read_status_static.restype = c_int
     lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
     lib.kd_workspace_size_batch.restype = c_sz
     lib.kd_decompose_batch.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
@@ -184,6 +190,17 @@ def kd_reconstruct_batch(mats, count, n, out_dtype, layout, workspace, ws_bytes,
 
 def kd_read_status(workspace, stream) -> int:
     return lib.kd_read_status(workspace, stream)
+
+
+def kd_decompose_static(w, dtype, layout, n, m, ld, sign_seed, iters, kmeans_iters, codes_u, codes_v, centres_u,
+                        centres_v, coeffs, u, vhat, resid, trace, stream) -> int:
+    return lib.kd_decompose_static(w, dtype, layout, n, m, ld, ctypes.c_uint64(int(sign_seed) & ((1 << 64) - 1)),
+                                   iters, kmeans_iters, codes_u, codes_v, centres_u, centres_v, coeffs, u, vhat,
+                                   resid, trace, stream)
+
+
+def kd_read_status_static(stream) -> int:
+    return lib.kd_read_status_static(stream)
 
 
 def kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream) -> int:

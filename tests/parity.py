@@ -33,6 +33,7 @@ TOL_FACTOR = 1e-5   # u, vhat, coefficients, centres
 TOL_RECON = 1e-6    # x = u + P vhat + r from device factors
 CODE_WINDOW = 1e-6  # near-boundary window, relative to a1 + a2
 CODE_FRAC = 1e-4    # at most 0.01 % of entries may differ, all inside the window
+R_RESOLVED = 1e-5   # residual norms compared where the oracle's ||r_k|| / ||x|| is at least this
 
 
 @dataclasses.dataclass
@@ -51,6 +52,14 @@ class ParityReport:
     code_near: int
     recon_err: float
     entries: int
+    # per-vector residual norms ||r_k||_2 / ||x||_2 (device, oracle) and the
+    # reconstruction-error contract E = ||W - W_hat||_F / ||W||_F (when measured)
+    r_gpu: np.ndarray = dataclasses.field(default=None, repr=False)
+    r_ora: np.ndarray = dataclasses.field(default=None, repr=False)
+    resid_err: float = 0.0
+    resid_ratio: float = 0.0
+    e_gpu: float = float("nan")
+    e_ora: float = float("nan")
 
     def check(self, code_budget: bool = True):
         """code_budget=False for degenerate inputs (constant vectors, single spikes)
@@ -130,20 +139,46 @@ def compare(x: np.ndarray, seed: int, iters: int, dev: dict, P_oracle=None, kmea
         outside += int((mism & ~near).sum())
 
     Pv = P(v_g)
-    recon = np.linalg.norm(x - u_g - Pv - r_g, axis=0) / np.where(np.linalg.norm(x, axis=0) > 0,
-                                                                  np.linalg.norm(x, axis=0), 1)
+    nx = np.linalg.norm(x, axis=0)
+    nx1 = np.where(nx > 0, nx, 1)
+    recon = np.linalg.norm(x - u_g - Pv - r_g, axis=0) / nx1
+    r_gpu = np.linalg.norm(r_g, axis=0) / nx1
+    r_ora = np.linalg.norm(d.r, axis=0) / nx1
+    resid_err, resid_ratio = residual_stats(r_gpu, r_ora)
+    e_gpu = e_ora = float("nan")
+    if "w_hat" in dev:
+        # App. C: the dequantised weight W_hat = U_q + P V_q; device from kd_reconstruct on
+        # its own codes and centres, oracle from its own (fp64, dense P)
+        wh_ora = ko.dequantise(code_u, cu) + P(ko.dequantise(code_v, cv))
+        nW = np.linalg.norm(x)
+        e_gpu = float(np.linalg.norm(x - dev["w_hat"].T.astype(np.float64)) / nW)
+        e_ora = float(np.linalg.norm(x - wh_ora) / nW)
     return ParityReport(n=N, m=M, hard=d.hard_mismatches + km_hard, ties=d.ties, tie_flips=d.tie_flips, u_err=u_err,
                         v_err=v_err, coef_err=coef_err, cent_err=cent_err, code_diff=diff,
                         code_diff_outside=outside, code_near=near_total, recon_err=float(recon.max()),
-                        entries=2 * N * M)
+                        entries=2 * N * M, r_gpu=r_gpu, r_ora=r_ora, resid_err=resid_err,
+                        resid_ratio=resid_ratio, e_gpu=e_gpu, e_ora=e_ora)
 
 
-def device_outputs(kd, w_dev, iters, seed, trace=True, layout="rows", kmeans_iters=0):
-    """Run kd_decompose with every optional output and return numpy arrays."""
+def residual_stats(r_gpu: np.ndarray, r_ora: np.ndarray):
+    """Per-vector residual norms (relative to ||x||), device against oracle.
+    Returns (largest relative disagreement among vectors whose oracle residual is
+    resolved in fp32, largest ratio r_gpu / r_ora over all vectors with r_ora > 0)."""
+    res = r_ora >= R_RESOLVED
+    err = float((np.abs(r_gpu[res] - r_ora[res]) / r_ora[res]).max()) if res.any() else 0.0
+    pos = r_ora > 0
+    ratio = float((r_gpu[pos] / r_ora[pos]).max()) if pos.any() else 0.0
+    return err, ratio
+
+
+def device_outputs(kd, w_dev, iters, seed, trace=True, layout="rows", kmeans_iters=0, w_hat=False):
+    """Run kd_decompose with every optional output and return numpy arrays; with
+    w_hat, also kd_reconstruct's fp32 W_hat from the device's codes and centres."""
     out = kd.decompose(w_dev, iters, seed, layout=layout, factors=True, coeffs=True, trace=trace,
                        kmeans_iters=kmeans_iters)
     n = out.u.shape[1]
     import torch
+    wh = kd.reconstruct(out, n, seed, dtype=torch.float32) if w_hat else None
     torch.cuda.synchronize()
     res = {
         "u": out.u.cpu().numpy(), "vhat": out.vhat.cpu().numpy(), "resid": out.resid.cpu().numpy(),
@@ -154,4 +189,6 @@ def device_outputs(kd, w_dev, iters, seed, trace=True, layout="rows", kmeans_ite
     }
     if trace:
         res["trace"] = out.trace.cpu().numpy()
+    if wh is not None:
+        res["w_hat"] = wh.cpu().numpy()
     return res

@@ -248,3 +248,28 @@ def test_batch_wrappers_validate_counts_on_the_host(kd):
         kd.reconstruct_batch([None] * (kd.KD_MAX_BATCH + 1), 256, list(range(kd.KD_MAX_BATCH + 1)))
     with pytest.raises(ValueError):
         kd.decompose_batch([None, None], 4, [1])
+
+
+def test_static_entry_checks_arguments_before_its_limit(kd):
+    """kd_decompose_static checks the caller's arguments in kd_decompose's order and
+    with its codes before applying its own length limit; none of these calls touches
+    the GPU (the array's address is resolved only after every check passed)."""
+    null = None
+    st = kd.kd_decompose_static
+    # a bad enum, a bad count or an unsupported length win over the length limit
+    assert st(16, 7, 0, 16384, 4, 16384, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_INVALID_ARG
+    assert st(16, 0, 0, 16384, 4, 16384, 0, -1, 0, 16, 16, 16, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_INVALID_ARG
+    assert st(16, 0, 0, 16382, 4, 16382, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_UNSUPPORTED_N
+    # ld too small, a null required output, an unaligned pointer
+    assert st(16, 0, 0, 11008, 4, 100, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_INVALID_ARG
+    assert st(16, 0, 0, 11008, 4, 11008, 0, 4, 0, 16, null, 16, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_INVALID_ARG
+    assert st(16, 0, 0, 11008, 4, 11008, 0, 4, 0, 16, 16, 18, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_INVALID_ARG
+    # valid arguments beyond the static array's limit
+    assert st(16, 0, 0, 11008, 4, 11008, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null,
+              null) == kd.KD_ERR_WORKSPACE

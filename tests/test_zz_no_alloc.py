@@ -4,7 +4,10 @@ on purpose; it must pass alone in a fresh process and after the other tests.
 
 Checked through the C ABI: two calls in a row (different vector lengths, so the
 shared static tables are rewritten between them) must reproduce kd_decompose with
-a caller workspace, and a vector length above the static limit is refused."""
+a caller workspace bit for bit (the same kernels and tables run on both paths), a
+repeated call must leave the device's free memory unchanged, a non-finite input
+must be reported by kd_read_status_static, and a vector length above the static
+limit is refused."""
 
 import ctypes
 
@@ -26,6 +29,8 @@ def env():
     lib.kd_decompose_static.argtypes = [vp, ctypes.c_int, ctypes.c_int, i64, i64, i64, ctypes.c_uint64,
                                         ctypes.c_int, ctypes.c_int] + [vp] * 10
     lib.kd_decompose_static.restype = ctypes.c_int
+    lib.kd_read_status_static.argtypes = [vp]
+    lib.kd_read_status_static.restype = ctypes.c_int
     return torch, kd, lib
 
 
@@ -56,12 +61,46 @@ def test_static_scratch_matches_workspace_path(env):
         got = _static(torch, kd, lib, w, 16, seed)
         ref = kd.decompose(w, 16, seed, factors=True, coeffs=True)
         torch.cuda.synchronize()
-        for k in ("codes_u", "codes_v", "centres_u", "centres_v", "coeffs"):
+        for k in ("codes_u", "codes_v", "centres_u", "centres_v", "coeffs", "u", "vhat", "resid"):
             assert torch.equal(got[k], getattr(ref, k)), (call, k)
-        for k in ("u", "vhat", "resid"):
-            a, b = got[k].double(), getattr(ref, k).double()
-            scale = b.abs().amax(dim=1, keepdim=True).clamp_min(1e-30)
-            assert ((a - b).abs() / scale).max().item() <= 1e-5, (call, k)
+        assert lib.kd_read_status_static(torch.cuda.current_stream().cuda_stream) == kd.KD_OK
+
+
+def test_static_call_allocates_nothing(env):
+    """A repeated call (its kernels already loaded by the first) must not change the
+    device's free memory: the scratch is the static array, nothing else is taken."""
+    torch, kd, lib = env
+    g = torch.Generator().manual_seed(7)
+    w = (torch.randn((12, 4096), generator=g) * 0.02).half().cuda()
+    first = _static(torch, kd, lib, w, 8, 3)
+    torch.cuda.synchronize()
+    free_before, _ = torch.cuda.mem_get_info()
+    seed, iters = 3, 8
+    m, n = w.shape
+    st = lib.kd_decompose_static(w.data_ptr(), kd.KD_F16, kd.KD_VEC_ROWS, n, m, n, seed, iters, 0,
+                                 first["codes_u"].data_ptr(), first["codes_v"].data_ptr(),
+                                 first["centres_u"].data_ptr(), first["centres_v"].data_ptr(),
+                                 first["coeffs"].data_ptr(), first["u"].data_ptr(), first["vhat"].data_ptr(),
+                                 first["resid"].data_ptr(), None, torch.cuda.current_stream().cuda_stream)
+    assert st == kd.KD_OK
+    assert lib.kd_read_status_static(torch.cuda.current_stream().cuda_stream) == kd.KD_OK
+    torch.cuda.synchronize()
+    free_after, _ = torch.cuda.mem_get_info()
+    assert free_after == free_before
+
+
+def test_static_status_reports_nonfinite_input(env):
+    """A NaN in the input sets the status word in the static array; the next call with
+    finite inputs clears it again."""
+    torch, kd, lib = env
+    w = (torch.arange(4 * 256, dtype=torch.float32).reshape(4, 256) * 1e-3 - 0.5).cuda()
+    bad = w.clone()
+    bad[1, 17] = float("nan")
+    stream = torch.cuda.current_stream().cuda_stream
+    _static(torch, kd, lib, bad, 4, 1)
+    assert lib.kd_read_status_static(stream) == kd.KD_ERR_NONFINITE
+    _static(torch, kd, lib, w, 4, 1)
+    assert lib.kd_read_status_static(stream) == kd.KD_OK
 
 
 def test_static_scratch_refuses_long_vectors(env):
