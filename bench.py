@@ -94,7 +94,7 @@ def flops_per_vector(n: int, iters: int) -> float:
 
 # sources the N = 4096 decompose kernel is built from (the profile's DRAM figures
 # stay valid while these are unchanged)
-DECOMPOSE_SOURCES = ("kd_math.cuh", "kd_xform.cuh", "kd_kernels.cuh", "kd_plans.cuh", "kd_launch.cuh", "kd_ops.h",
+DECOMPOSE_SOURCES = ("kd_math.cuh", "kd_xform.cuh", "kd_kernels.cuh", "kd_bulk.cuh", "kd_plans.cuh", "kd_launch.cuh", "kd_ops.h",
                      "kd_plan_4096.cu")
 
 

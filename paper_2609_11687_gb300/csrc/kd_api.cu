@@ -153,6 +153,13 @@ bool outputs_aligned(const void* w, int dtype, const void* codes_u, const void* 
 }
 bool valid_layout(int l) { return l == KD_VEC_ROWS || l == KD_VEC_COLUMNS; }
 
+// A matrix whose vectors are contiguous rows starting on 16-byte boundaries: the
+// decomposition stages each pair's rows into shared memory with bulk copies.
+bool rows_bulk_ok(const void* w, int dtype, int layout, int64_t n, int64_t ld) {
+  const int64_t esz = dtype == KD_F32 ? 4 : 2;
+  return layout == KD_VEC_ROWS && aligned_to(w, 16) && (ld * esz) % 16 == 0 && (n * esz) % 16 == 0;
+}
+
 }  // namespace
 
 int check_decompose_args(const void* w, int dtype, int layout, int64_t n, int64_t m, int64_t ld, int iters,
@@ -251,6 +258,7 @@ kd_status kd_decompose(const void* w, kd_dtype dtype, kd_layout layout, int64_t 
   p.status = reinterpret_cast<uint32_t*>(b + L.status);
   p.uslots = ops->u_in_gmem ? reinterpret_cast<float2*>(b + L.uslots) : nullptr;
   p.npairs = (m + 1) / 2;
+  p.bulk = rows_bulk_ok(w, dtype, layout, n, ld) ? 1 : 0;
   const int ctas = max_decompose_ctas(ops);
   if (ctas <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, ctas);
@@ -331,6 +339,9 @@ kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, k
   p.status = reinterpret_cast<uint32_t*>(b + L.status);
   p.uslots = ops->u_in_gmem ? reinterpret_cast<float2*>(b + L.uslots) : nullptr;
   p.npairs = npairs;
+  p.bulk = 1;
+  for (int i = 0; i < count; ++i)
+    if (mats[i].m > 0 && !rows_bulk_ok(mats[i].w, dtype, layout, n, mats[i].ld)) p.bulk = 0;
   const int ctas = max_decompose_ctas(ops);
   if (ctas <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, ctas);

@@ -35,6 +35,7 @@
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
+#include "kd_bulk.cuh"
 #include "kd_math.cuh"
 #include "kd_xform.cuh"
 
@@ -187,6 +188,9 @@ struct DecParams {
   uint32_t* status;
   float2* uslots;
   int64_t npairs;
+  // 1: every vector of the launch is a contiguous, 16-byte aligned row (KD_VEC_ROWS,
+  // w and ld * element size multiples of 16 bytes): pairs are staged by bulk copies
+  int bulk;
 };
 
 // Several matrices of one vector length in one launch (kd_decompose_batch): their
@@ -237,6 +241,22 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
   if constexpr (PL::UMODE == UGMEM) uslot = p.uslots + ((int64_t)blockIdx.x * PL::Q + team) * N;
   if constexpr (PL::UMODE == USMEM) uslot = red + PL::RED;
 
+  static_assert(PL::SMEM_TW % 16 == 0 && PL::TEAM % 2 == 0, "team buffers must start 16-byte aligned");
+  // Staged input (p.bulk): the pair's two rows land in the team's exchange buffer by
+  // bulk copy (16-byte aligned rows, completion on the team's mbarrier), and every
+  // thread reads its elements in Makhoul order from there; the same staging re-reads
+  // x after the last block.  Otherwise the elements are gathered from global memory.
+  uint64_t* mbar = reinterpret_cast<uint64_t*>(buf + PL::BUF + PL::RED + PL::USL);
+  uint32_t mphase = 0;
+  if (p.bulk) {
+    if (lt == 0) {
+      mbar_init(mbar, 1);
+      mbar_init_fence();
+    }
+    __syncthreads();
+  }
+  const int esz = p.dtype == DT_F32 ? 4 : 2;
+
   int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
@@ -261,14 +281,70 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
     const bool hasB = (colA + 1) < m_in;
     const int64_t colB = hasB ? colA + 1 : colA;
 
+    // Bulk-copy both rows of the pair into buf (free: every reader of the previous
+    // use passed a team barrier); false if the copy did not land in time, decided for
+    // the whole CTA so that its barriers stay uniform.
+    auto stage_rows = [&](bool prefetch_next) -> bool {
+      const uint32_t rb = (uint32_t)(N * esz);
+      if (lt == 0) {
+        const char* w0 = static_cast<const char*>(w_in());
+        fence_proxy_async_smem();  // earlier generic accesses to buf before the copy's writes
+        mbar_arrive_expect_tx(mbar, hasB ? 2 * rb : rb);
+        bulk_copy_g2s(buf, w0 + colA * ld_in() * esz, rb, mbar);
+        if (hasB) bulk_copy_g2s(reinterpret_cast<char*>(buf) + rb, w0 + colB * ld_in() * esz, rb, mbar);
+        // the rows this team takes next, into L2 while this pair is decomposed
+        const int64_t nxt = pair + (int64_t)gridDim.x * PL::Q;
+        if (prefetch_next && nxt < p.npairs) {
+          int mn = 0;
+          int64_t pn = nxt;
+          if (batched) {
+            while (mn + 1 < bp.count && pn >= bp.mat[mn + 1].pair0) ++mn;
+            pn -= bp.mat[mn].pair0;
+          }
+          const char* wn = static_cast<const char*>(batched ? bp.mat[mn].w : p.w);
+          const int64_t ldn = batched ? bp.mat[mn].ld : p.ld;
+          const int64_t mm = batched ? bp.mat[mn].m : p.m;
+          bulk_prefetch_l2(wn + 2 * pn * ldn * esz, rb);
+          if (2 * pn + 1 < mm) bulk_prefetch_l2(wn + (2 * pn + 1) * ldn * esz, rb);
+        }
+      }
+      const bool ok = mbar_wait_bounded(mbar, mphase);
+      mphase ^= 1u;
+      if (__syncthreads_or(!ok)) {
+        if (lt == 0) {
+          atomicOr(p.status, 2u);
+          mbar_wait_bounded(mbar, mphase ^ 1u);  // let the copy land before the CTA leaves
+        }
+        __syncthreads();
+        return false;
+      }
+      return true;
+    };
+    // element nat of staged row c (0 = vector A, 1 = vector B)
+    auto staged = [&](int c, int nat) -> float {
+      const char* row = reinterpret_cast<const char*>(buf) + c * N * esz;
+      if (p.dtype == DT_F32) return reinterpret_cast<const float*>(row)[nat];
+      if (p.dtype == DT_F16) return __half2float(reinterpret_cast<const __half*>(row)[nat]);
+      return __bfloat162float(reinterpret_cast<const __nv_bfloat16*>(row)[nat]);
+    };
+
     // ---- load the pair in Makhoul order: position lt + j*T ----
+    // (staged: the first greedy step's team reduction, or the transform's opening
+    // barrier for single-warp teams, orders these reads before buf is written again)
     float2 r[E];
     float2 acc = make_float2(0.f, 0.f);
+    if (p.bulk && !stage_rows(true)) return;
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
-      const float a = load_elem(w_in(), p.dtype, elem_index(p.layout, colA, nat, ld_in()));
-      const float b = hasB ? load_elem(w_in(), p.dtype, elem_index(p.layout, colB, nat, ld_in())) : 0.f;
+      float a, b;
+      if (p.bulk) {
+        a = staged(0, nat);
+        b = hasB ? staged(1, nat) : 0.f;
+      } else {
+        a = load_elem(w_in(), p.dtype, elem_index(p.layout, colA, nat, ld_in()));
+        b = hasB ? load_elem(w_in(), p.dtype, elem_index(p.layout, colB, nat, ld_in())) : 0.f;
+      }
       r[j] = make_float2(a, b);
       acc.x = __fadd_rn(acc.x, fabsf(a));
       acc.y = __fadd_rn(acc.y, fabsf(b));
@@ -379,12 +455,21 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
             if (hasB) p.resid[colB * N + nat] = __fmul_rn(r[j].y, isB);
           }
         }
+        if (p.bulk) {
+          team_sync<PL>();  // the last transform's readers of buf are done
+          if (!stage_rows(false)) return;
+        }
 #pragma unroll
         for (int j = 0; j < E; ++j) {
           const int nat = nat_of<N>(lt + j * T);
-          const float a = __fmul_rn(load_elem(w_in(), p.dtype, elem_index(p.layout, colA, nat, ld_in())), scA);
-          const float b =
-              hasB ? __fmul_rn(load_elem(w_in(), p.dtype, elem_index(p.layout, colB, nat, ld_in())), scB) : 0.f;
+          float a, b;
+          if (p.bulk) {
+            a = __fmul_rn(staged(0, nat), scA);
+            b = hasB ? __fmul_rn(staged(1, nat), scB) : 0.f;
+          } else {
+            a = __fmul_rn(load_elem(w_in(), p.dtype, elem_index(p.layout, colA, nat, ld_in())), scA);
+            b = hasB ? __fmul_rn(load_elem(w_in(), p.dtype, elem_index(p.layout, colB, nat, ld_in())), scB) : 0.f;
+          }
           const float2 uj = u_at(j);
           r[j] = make_float2(__fsub_rn(__fsub_rn(a, uj.x), r[j].x), __fsub_rn(__fsub_rn(b, uj.y), r[j].y));
         }
@@ -393,7 +478,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) decompose_kernel(DecPar
           for (int j = 0; j < E; ++j) r[j] = make_float2(0.f, 0.f);
           break;
         }
-        team_sync<PL>();  // the last transform's readers of buf are done
+        team_sync<PL>();  // the last transform's readers of buf (or of the staged x) are done
       } else if ((hb & 1) == 0) {
         // two greedy steps from Q_N (update u).  u outside registers (shared memory,
         // or the workspace slot for the longest vectors) is updated in place by both
@@ -622,7 +707,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyPar
   const int lt = threadIdx.x - team * T;
   const float2* tw;
   float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
-  Xform<PL> xf;
+  Xform<PL, false> xf;  // scalar roots: no registers to spare for constant pairs
   xf.init(buf, tw, p.eps, lt);
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
@@ -693,7 +778,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
   const int lt = threadIdx.x - team * T;
   const float2* tw;
   float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
-  Xform<PL> xf;
+  Xform<PL, false> xf;  // scalar roots: no registers to spare for constant pairs
   xf.init(buf, tw, p.eps, lt);
   int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {

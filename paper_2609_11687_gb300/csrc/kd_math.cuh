@@ -85,6 +85,8 @@ __device__ __forceinline__ float2 cadd(float2 a, float2 b) {
 __device__ __forceinline__ float2 csub(float2 a, float2 b) {
   return __ffma2_rn(b, make_float2(-1.f, -1.f), a);
 }
+// Complex products stay scalar: a packed form needs a sign-flipped copy of one
+// operand, one more FMA-pipe instruction than the four scalar ones (measured).
 // a * b
 __device__ __forceinline__ float2 cmul(float2 a, float2 b) {
   return make_float2(__fmaf_rn(a.x, b.x, __fmul_rn(-a.y, b.y)),
@@ -110,10 +112,16 @@ __device__ __forceinline__ float2 add_ib(float2 a, float2 b) {
 __device__ __forceinline__ float2 sub_ib(float2 a, float2 b) {
   return make_float2(__fadd_rn(a.x, b.y), __fsub_rn(a.y, b.x));
 }
+// swapped pair: packed FP32x2 instructions read either half of a register pair for
+// either lane, so (a.y, a.x) as an operand costs no instruction (measured on sm_103a)
+__device__ __forceinline__ float2 swp(float2 a) { return make_float2(a.y, a.x); }
 
 // Multiply by the compile-time root W_R^E = exp(DIR * 2 pi i E / R), DIR = -1 forward.
 // Quarter turns are exact; eighth turns use one constant; others a full product.
-template <int DIR, long long E, long long R>
+// PK selects packed forms on the swapped pair (two FP32x2 instructions instead of
+// four scalar ones, the same FMA-pipe cycles): fewer issue slots, but the constant
+// pairs occupy registers, so a plan opts in only where registers are to spare.
+template <int DIR, long long E, long long R, bool PK = false>
 __device__ __forceinline__ float2 mul_root(float2 a) {
   constexpr long long e = kd_mod(E, R);
   if constexpr (e == 0) {
@@ -131,9 +139,12 @@ __device__ __forceinline__ float2 mul_root(float2 a) {
     // exp(i*pi*oo/4) = (c, s) with |c| = |s| = h
     constexpr float c = (oo == 1 || oo == 7) ? h : -h;
     constexpr float s = (oo == 1 || oo == 3) ? h : -h;
-    // (a.x + i a.y)(c + i s) = (c a.x - s a.y) + i (s a.x + c a.y)
-    // c*(a.x - (s/c) a.y), c*(a.y + (s/c) a.x) with s/c = +-1 exact
-    if constexpr ((c > 0) == (s > 0)) {
+    // (a.x + i a.y)(c + i s) = c (a.x - (s/c) a.y, a.y + (s/c) a.x) with s/c = +-1 exact:
+    // one packed FMA on the swapped pair, one packed multiply
+    if constexpr (PK) {
+      constexpr float q = (c > 0) == (s > 0) ? 1.f : -1.f;
+      return __fmul2_rn(__ffma2_rn(swp(a), make_float2(-q, q), a), make_float2(c, c));
+    } else if constexpr ((c > 0) == (s > 0)) {
       return make_float2(__fmul_rn(c, __fsub_rn(a.x, a.y)), __fmul_rn(c, __fadd_rn(a.y, a.x)));
     } else {
       return make_float2(__fmul_rn(c, __fadd_rn(a.x, a.y)), __fmul_rn(c, __fsub_rn(a.y, a.x)));
@@ -141,7 +152,12 @@ __device__ __forceinline__ float2 mul_root(float2 a) {
   } else {
     constexpr float c = (float)cos2pi(e, R);
     constexpr float s = (float)((DIR > 0 ? 1.0 : -1.0) * sin2pi(e, R));
-    return make_float2(__fmaf_rn(a.x, c, __fmul_rn(-a.y, s)), __fmaf_rn(a.x, s, __fmul_rn(a.y, c)));
+    if constexpr (PK) {
+      // a (c, c) + swap(a) (-s, s)
+      return __ffma2_rn(swp(a), make_float2(-s, s), __fmul2_rn(a, make_float2(c, c)));
+    } else {
+      return make_float2(__fmaf_rn(a.x, c, __fmul_rn(-a.y, s)), __fmaf_rn(a.x, s, __fmul_rn(a.y, c)));
+    }
   }
 }
 
@@ -169,17 +185,17 @@ struct SmallestFactor {
                              : (R % 5 == 0) ? 5 : (R % 7 == 0) ? 7 : R;
 };
 
-template <int R, int DIR>
+template <int R, int DIR, bool PK = false>
 struct Dft;
 
-template <int DIR>
-struct Dft<1, DIR> {
+template <int DIR, bool PK>
+struct Dft<1, DIR, PK> {
   template <class A>
   __device__ __forceinline__ static void run(A&) {}
 };
 
-template <int DIR>
-struct Dft<2, DIR> {
+template <int DIR, bool PK>
+struct Dft<2, DIR, PK> {
   template <class A>
   __device__ __forceinline__ static void run(A& v) {
     float2 a = v[0], b = v[1];
@@ -188,8 +204,8 @@ struct Dft<2, DIR> {
   }
 };
 
-template <int DIR>
-struct Dft<4, DIR> {
+template <int DIR, bool PK>
+struct Dft<4, DIR, PK> {
   template <class A>
   __device__ __forceinline__ static void run(A& v) {
     float2 s02 = cadd(v[0], v[2]), d02 = csub(v[0], v[2]);
@@ -299,7 +315,7 @@ KD_HD constexpr bool kd_is_big_prime() {
 //   n = B*n1 + n2 ; k = k1 + A*k2
 //   step 1: for each n2, size-A DFT over n1 -> k1 ; multiply by W_R^{n2*k1}
 //   step 2: for each k1, size-B DFT over n2 -> k2.
-template <int R, int DIR>
+template <int R, int DIR, bool PK>
 struct DftComposite {
   static constexpr int A = SmallestFactor<R>::value;
   static constexpr int B = R / A;
@@ -311,10 +327,10 @@ struct DftComposite {
       float2 s[A];
 #pragma unroll
       for (int n1 = 0; n1 < A; ++n1) s[n1] = v[B * n1 + N2];
-      Dft<A, DIR>::run(s);
+      Dft<A, DIR, PK>::run(s);
       static_for<0, A>([&](auto k1c) {
         constexpr int K1 = decltype(k1c)::value;
-        t[K1 * B + N2] = mul_root<DIR, (long long)N2 * K1, R>(s[K1]);
+        t[K1 * B + N2] = mul_root<DIR, (long long)N2 * K1, R, PK>(s[K1]);
       });
     });
 #pragma unroll
@@ -322,21 +338,21 @@ struct DftComposite {
       float2 s[B];
 #pragma unroll
       for (int n2 = 0; n2 < B; ++n2) s[n2] = t[k1 * B + n2];
-      Dft<B, DIR>::run(s);
+      Dft<B, DIR, PK>::run(s);
 #pragma unroll
       for (int k2 = 0; k2 < B; ++k2) v[k1 + A * k2] = s[k2];
     }
   }
 };
 
-template <int R, int DIR>
+template <int R, int DIR, bool PK>
 struct Dft {
   template <class A>
   __device__ __forceinline__ static void run(A& v) {
     if constexpr (SmallestFactor<R>::value == R) {
       DftPrime<R, DIR>::run(v);
     } else {
-      DftComposite<R, DIR>::run(v);
+      DftComposite<R, DIR, PK>::run(v);
     }
   }
 };

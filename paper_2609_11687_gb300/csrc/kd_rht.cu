@@ -31,6 +31,7 @@
 #include <cuda_fp16.h>
 
 #include "kashin.h"
+#include "kd_bulk.cuh"
 #include "kd_math.cuh"
 
 namespace kd {
@@ -52,7 +53,6 @@ struct RhtParams {
 };
 
 constexpr uint32_t kRhtErrTimeout = 1u;           // a stage's bulk copy did not complete in time
-constexpr long long kWaitCycles = 2000000000ll;  // ~1 s at the maximum SM clock
 
 KD_HD constexpr int rht_threads(int log_b) { return ((1 << log_b) / 16) > 256 ? ((1 << log_b) / 16) : 256; }
 // resident CTAs per SM the register budget is sized for (1024 threads: 64 registers each)
@@ -362,56 +362,6 @@ __global__ void __launch_bounds__(rht_threads(LOG_B)) rht_kernel(RhtParams p) {
 // ---------------------------------------------------------------------------
 // Bulk-copy staged variant
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ uint32_t smem_u32(const void* ptr) {
-  return (uint32_t)__cvta_generic_to_shared(ptr);
-}
-
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_init_fence() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t done;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(done)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return done != 0;
-}
-
-// waits for the phase of `bar` with this parity; false once kWaitCycles have passed
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
-  const long long t0 = clock64();
-  while (!mbar_try_wait(bar, parity)) {
-    if (clock64() - t0 > kWaitCycles) return false;
-  }
-  return true;
-}
-
-// global -> shared bulk copy; completion is counted on `bar` (bytes)
-__device__ __forceinline__ void bulk_copy_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                   smem_u32(dst)),
-               "l"(src), "r"(bytes), "r"(smem_u32(bar))
-               : "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async_smem() {
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
 template <int LOG_B>
 KD_HD constexpr int rht_stages() { return LOG_B >= 14 ? 2 : 3; }
 

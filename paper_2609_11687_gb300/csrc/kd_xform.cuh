@@ -84,6 +84,14 @@ __device__ __forceinline__ float4 ld_tw4(const float2* p) {
   return v;
 }
 
+// Plans that apply the DFTs' constant roots in packed FP32x2 form (kd_math.cuh
+// mul_root): opted in per plan (kd_plans.cuh) where the registers allow it and it
+// measured faster.
+template <class PL>
+struct PackedRoots {
+  static constexpr bool value = false;
+};
+
 template <int N_, int T_, int Q_, int UMODE_, int MINB_, int... Rs>
 struct Plan {
   static constexpr int N = N_;
@@ -105,6 +113,7 @@ struct Plan {
   // 16-value reduction of the k-means refinement (16 (NW + 1) floats = 8 (NW + 1) float2)
   static constexpr int RED = (4 * NW > 8 * (NW + 1)) ? 4 * NW : 8 * (NW + 1);
   static constexpr int USL = (UMODE_ == 2) ? N : 0;            // float2 slots of u per team (shared)
+  static constexpr int MBS = 2;  // float2 slots holding the team's mbarrier (bulk-copy staging)
   // M in registers: one last-pass group per thread, partner at lane ^ HALF
   static constexpr bool PAIRED = (RL == E) && (N / RL == T);
   static constexpr int HALF = (T < 32 ? T : 32) / 2;
@@ -125,7 +134,7 @@ struct Plan {
   static constexpr int TWN = tw_off(NP - 1);
 
   // stage the table in shared memory when MINB CTAs per SM still fit
-  static constexpr int TEAM = BUF + RED + USL;  // float2 slots of shared memory per team
+  static constexpr int TEAM = BUF + RED + USL + MBS;  // float2 slots of shared memory per team
   static constexpr bool TW_SMEM = (size_t)TWN * 8 + (size_t)Q * TEAM * 8 <= (size_t)(227 * 1024) / MINB - 1024;
   static constexpr size_t SMEM_TW = TW_SMEM ? (size_t)TWN * sizeof(float2) : 0;
   // paired twiddle layout (table staged in shared memory, every twiddled pass of even
@@ -234,7 +243,8 @@ __device__ __forceinline__ int rest_of_slot(int s) {
 }
 
 // ---------------------------------------------------------------------------
-template <class PL>
+// PKX: packed constant roots in the DFTs (the plan's choice by default)
+template <class PL, bool PKX = PackedRoots<PL>::value>
 struct Xform {
   static constexpr int N = PL::N, T = PL::T, E = PL::E, NP = PL::NP;
   float2* buf;                 // team's padded exchange buffer (shared)
@@ -245,6 +255,7 @@ struct Xform {
   Mask ek, em;                 // eps_k < 0 / eps_{-k} < 0 for each owned frequency (bit index)
   Mask dm;                     // ek ^ em: frequencies whose M takes the partner value
   static constexpr float kInvN = 1.0f / (float)N;
+  static constexpr bool PK = PKX;
   // Warp-local middle passes (16 x 16 x 16 with 256 threads): after pass 0 the
   // vector falls into 16 blocks of 256 slots (one per pass-0 output digit b), and the
   // M partner of every last-pass group of block b lies in block 16 - b (blocks 0 and
@@ -338,7 +349,7 @@ struct Xform {
   template <long long RNUM, long long RDEN, int BIT>
   __device__ __forceinline__ float2 mfreq(float2 a, float2 b) const {
     // exp(i pi k / N) = cw * exp(i pi RNUM / RDEN)
-    const float2 wk = mul_root<+1, RNUM, 2 * RDEN>(cw);
+    const float2 wk = mul_root<+1, RNUM, 2 * RDEN, PK>(cw);
     const float2 t = cmul(b, wk);
     const bool diff = (dm >> BIT) & 1u;
     const float2 sel = diff ? t : a;
@@ -385,7 +396,7 @@ struct Xform {
                                 buf[a0<K>()] = x;
                               });
     } else {
-      Dft<E, -1>::run(v);
+      Dft<E, -1, PK>::run(v);
       twiddle<0, T, E, -1>(v, lt);
       static_for<0, E>([&](auto jc) { buf[a0<decltype(jc)::value>()] = v[decltype(jc)::value]; });
     }
@@ -407,7 +418,7 @@ struct Xform {
     } else {
       static_for<0, E>([&](auto jc) { v[decltype(jc)::value] = buf[a0<decltype(jc)::value>()]; });
       twiddle<0, T, E, +1>(v, lt);
-      Dft<E, +1>::run(v);
+      Dft<E, +1, PK>::run(v);
     }
   }
 
@@ -433,11 +444,11 @@ struct Xform {
 #pragma unroll
       for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
       if constexpr (DIR < 0) {
-        Dft<R, -1>::run(v);
+        Dft<R, -1, PK>::run(v);
         if constexpr (!LAST) twiddle<I, S, R, -1>(v, np);
       } else {
         if constexpr (!LAST) twiddle<I, S, R, +1>(v, np);
-        Dft<R, +1>::run(v);
+        Dft<R, +1, PK>::run(v);
       }
 #pragma unroll
       for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
@@ -445,7 +456,10 @@ struct Xform {
     }
   }
 
-  // paired last pass: forward DFT of own group, M with the partner lane, inverse DFT
+  // paired last pass: forward DFT of own group, M with the partner lane, inverse DFT.
+  // M runs in place, two mirrored indices (KP, R-1-KP) at a time: the partner lane's
+  // value for index KP is its v[R-1-KP], so each step exchanges both of a mirrored
+  // pair's sources before overwriting them (no second array of R values is live).
   __device__ __forceinline__ void last_paired() {
     constexpr int R = PL::RL;
     constexpr int H = PL::HALF;
@@ -456,24 +470,42 @@ struct Xform {
     float2 v[R];
 #pragma unroll
     for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
-    Dft<R, -1>::run(v);
-    float2 o[R];
+    Dft<R, -1, PK>::run(v);
     // Only the warp holding groups 0 and N/(2 RL) (self-paired) needs the local-value
     // selects; every other warp takes the shuffle-only path (warp-uniform branch).
+    // Group 0 pairs index KP with its own (R - KP) % R, which the in-place order may
+    // already have overwritten: its lane keeps the transformed values in its own slots.
     auto body = [&](auto slowc) {
       constexpr bool SLOW = decltype(slowc)::value;
-      static_for<0, R>([&](auto kk) {
-        constexpr int KP = decltype(kk)::value;
-        const float2 src = v[R - 1 - KP];
-        float2 q;
-        q.x = __shfl_xor_sync(0xffffffffu, src.x, H);
-        q.y = __shfl_xor_sync(0xffffffffu, src.y, H);
+      if constexpr (SLOW) {
+        if (self == 1) {
+#pragma unroll
+          for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
+        }
+      }
+      static_for<0, R / 2>([&](auto kk) {
+        constexpr int K1 = decltype(kk)::value;
+        constexpr int K2 = R - 1 - K1;
+        const float2 s1 = v[K2], s2 = v[K1];
+        float2 q1, q2;
+        q1.x = __shfl_xor_sync(0xffffffffu, s1.x, H);
+        q1.y = __shfl_xor_sync(0xffffffffu, s1.y, H);
+        q2.x = __shfl_xor_sync(0xffffffffu, s2.x, H);
+        q2.y = __shfl_xor_sync(0xffffffffu, s2.y, H);
         if constexpr (SLOW) {
-          if (self == 1) q = v[(R - KP) % R];
-          else if (self == 2) q = src;
+          if (self == 1) {
+            q1 = buf[addr((R - K1) % R)];
+            q2 = buf[addr((R - K2) % R)];
+          } else if (self == 2) {
+            q1 = s1;
+            q2 = s2;
+          }
         }
         // k = K + (N/R) KP: exp(i pi k/N) = exp(i pi K/N) exp(i pi KP/R)
-        o[KP] = mfreq<KP, R, KP>(v[KP], q);
+        const float2 o1 = mfreq<K1, R, K1>(s2, q1);
+        const float2 o2 = mfreq<K2, R, K2>(s1, q2);
+        v[K1] = o1;
+        v[K2] = o2;
       });
     };
     if (__any_sync(0xffffffffu, self != 0)) {
@@ -481,9 +513,9 @@ struct Xform {
     } else {
       body(std::false_type{});
     }
-    Dft<R, +1>::run(o);
+    Dft<R, +1, PK>::run(v);
 #pragma unroll
-    for (int j = 0; j < R; ++j) buf[addr(j)] = o[j];
+    for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
   }
 
   // slot-order M (own slots lt + T r, partners from constants); v is scratch
