@@ -634,93 +634,74 @@ def measure_refinement(kd, torch, layer, outs, wss, iters, stream, ndom):
 
 
 def run_e2e(kd, torch, layer, outs, wss, iters, args, stream, dist, world):
-    """Same metric through the C ABI with host buffers: every step copies the
-    layer's fp16 weights from pinned host memory and reads codes + centres back.
-    The matrices of one vector length form a group that goes out as one
-    kd_decompose_batch (as in the timed region); uploads, decompositions and
-    downloads run on three streams with two device copies of every group's inputs,
-    so one group uploads while another decomposes."""
+    """Same metric through the library's host-buffer entry point: every step, for
+    each vector length, one kd_decompose_batch_host call uploads that group's fp16
+    weights from pinned host memory, decomposes them in one batched launch and reads
+    the codes and centres back into pinned host memory, all on one stream.  Two slots
+    per group (stream, device staging, workspace, host outputs) alternate between
+    steps, so one step's copies overlap the other slot's decomposition."""
     host_in = [(s, w.cpu().pin_memory()) for s, w in layer]
     groups = {}
     for i, (s, _) in enumerate(layer):
         groups.setdefault(s.N, []).append(i)
-    gorder = list(groups)
-    wsb = {n_: kd.Workspace(n_, stream.device, count=len(ix)) for n_, ix in groups.items()}
-    slots = {n_: [[torch.empty_like(host_in[i][1], device=stream.device) for i in ix] for _ in range(2)]
-             for n_, ix in groups.items()}
-    dev_out = [kd.Decomposed(
-        codes_u=torch.empty_like(o.codes_u), codes_v=torch.empty_like(o.codes_v),
-        centres_u=torch.empty_like(o.centres_u), centres_v=torch.empty_like(o.centres_v),
-        coeffs=None, u=None, vhat=None, resid=None, trace=None) for o in outs]
-    host_out = [tuple(torch.empty(t.shape, dtype=t.dtype).pin_memory()
-                      for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v)) for o in dev_out]
+    slots = {}
+    for n_, ix in groups.items():
+        ws_h = [host_in[i][1] for i in ix]
+        nbytes = kd.staging_size_host(ws_h)
+        slots[n_] = [{"stream": torch.cuda.Stream(device=stream.device),
+                      "staging": torch.empty(nbytes, dtype=torch.uint8, device=stream.device),
+                      "ws": kd.Workspace(n_, stream.device, count=len(ix)),
+                      "outs": [kd.host_outputs(host_in[i][1].shape[0], n_) for i in ix]} for _ in range(2)]
     h2d = sum(w.numel() * w.element_size() for _, w in host_in)
-    d2h = sum(t.numel() * t.element_size() for o in dev_out for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v))
-    up = torch.cuda.Stream(device=stream.device)
-    down = torch.cuda.Stream(device=stream.device)
-    freed = {n_: [None, None] for n_ in groups}   # the launch that last read that input copy is done
-    use = {n_: 0 for n_ in groups}
-    read = {n_: None for n_ in groups}            # the group's outputs reached the host
+    d2h = sum(t.numel() * t.element_size() for o in outs for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v))
+    count = [0]
 
     def step():
-        for n_ in gorder:
-            ix = groups[n_]
-            k = use[n_] % 2
-            use[n_] += 1
-            dws = slots[n_][k]
-            with torch.cuda.stream(up):
-                if freed[n_][k] is not None:
-                    up.wait_event(freed[n_][k])
-                for i, dw in zip(ix, dws):
-                    dw.copy_(host_in[i][1], non_blocking=True)
-                loaded = torch.cuda.Event()
-                loaded.record(up)
-            stream.wait_event(loaded)
-            if read[n_] is not None:
-                stream.wait_event(read[n_])
-            kd.decompose_batch(dws, iters, [host_in[i][0].sign_seed for i in ix], workspace=wsb[n_],
-                               outs=[dev_out[i] for i in ix], stream=stream, kmeans_iters=args.kmeans_iters)
-            done = torch.cuda.Event()
-            done.record(stream)
-            freed[n_][k] = done
-            with torch.cuda.stream(down):
-                down.wait_event(done)
-                for i in ix:
-                    o = dev_out[i]
-                    for h, t in zip(host_out[i], (o.codes_u, o.codes_v, o.centres_u, o.centres_v)):
-                        h.copy_(t, non_blocking=True)
-                read[n_] = torch.cuda.Event()
-                read[n_].record(down)
+        k = count[0] % 2
+        count[0] += 1
+        for n_, ix in groups.items():
+            sl = slots[n_][k]
+            kd.decompose_batch_host([host_in[i][1] for i in ix], iters, [host_in[i][0].sign_seed for i in ix],
+                                    sl["outs"], sl["staging"], sl["ws"], stream=sl["stream"],
+                                    kmeans_iters=args.kmeans_iters)
 
-    def drain():
-        fin = torch.cuda.Event()
-        fin.record(down)
-        stream.wait_event(fin)
-
+    all_streams = [sl["stream"] for v in slots.values() for sl in v]
     for _ in range(2):
         step()
-    drain()
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     a = torch.cuda.Event(enable_timing=True)
     b = torch.cuda.Event(enable_timing=True)
-    n = max(3, args.steps // 4)
+    n = max(5, args.steps)
     a.record(stream)
-    up.wait_event(a)
-    down.wait_event(a)
+    for st in all_streams:
+        st.wait_event(a)
     for _ in range(n):
         step()
-    drain()
+    for st in all_streams:
+        e = torch.cuda.Event()
+        e.record(st)
+        stream.wait_event(e)
     b.record(stream)
     torch.cuda.synchronize()
+    # the host copies of the last step equal a device-resident run of the same layer
+    last = (count[0] - 1) % 2
+    for n_, ix in groups.items():
+        ref = kd.decompose_batch([host_in[i][1].to(stream.device) for i in ix], iters,
+                                 [host_in[i][0].sign_seed for i in ix], stream=stream, kmeans_iters=args.kmeans_iters)
+        torch.cuda.synchronize()
+        for r, o in zip(ref, slots[n_][last]["outs"]):
+            if not (torch.equal(o.codes_u, r.codes_u.cpu()) and torch.equal(o.centres_v, r.centres_v.cpu())):
+                raise RuntimeError("e2e host outputs differ from the device-resident run")
     from paper_2609_11687_gb300 import shard
     params = sum(s.params for s, _ in layer)
     ms, total = shard.aggregate(a.elapsed_time(b), n * params)
     return {"value": round(total / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": n,
-            "pipeline": "per vector length: H2D, one batched decompose and D2H on three streams, two copies of "
-                        "the inputs"}
+            "pipeline": "kd_decompose_batch_host per vector length (H2D from pinned host memory, one batched "
+                        "decompose, D2H of codes and centres, all on one stream), two alternating slots per "
+                        "length on their own streams"}
 
 
 # ---------------------------------------------------------------------------

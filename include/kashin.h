@@ -197,6 +197,49 @@ size_t kd_workspace_size_batch(int64_t n, int count);
 kd_status kd_decompose_batch(const kd_matrix* mats, int count, kd_dtype dtype, kd_layout layout, int64_t n,
                              int iters, int kmeans_iters, void* workspace, size_t ws_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * kd_decompose_batch from HOST memory to HOST memory: the end-to-end call of a caller
+ * that holds the weights on the host (Algorithm 1 and the 2-bit coding, as
+ * kd_decompose_batch).  Every pointer in the descriptors is HOST memory; pinned memory
+ * (cudaHostAlloc / cudaHostRegister) lets the copies run asynchronously, pageable
+ * memory makes them synchronous.  On `stream`, in order: one host-to-device copy per
+ * matrix input into `staging`, the batched decomposition, one device-to-host copy per
+ * output.  The call returns once this is enqueued; the host outputs are valid after
+ * the stream synchronises.  The host inputs must stay unchanged and the outputs
+ * untouched until then.  Several calls may be in flight on different streams, each
+ * with its own staging and workspace.
+ *
+ *   mats      HOST array of `count` descriptors (1 <= count <= KD_MAX_BATCH), read
+ *             during the call: w as kd_decompose's input (m vectors, layout and ld; the
+ *             whole m x ld block (KD_VEC_ROWS) or n x ld block (KD_VEC_COLUMNS) is
+ *             copied), codes_u, codes_v (m x ceil(n/16) uint32), centres_u, centres_v
+ *             (m x 4 fp32) required when m > 0, coeffs (m x 4) optional (NULL).
+ *   staging   device memory, 256-byte aligned, at least kd_staging_size_host() bytes:
+ *             the inputs and outputs on the device.  The library allocates nothing.
+ *   workspace at least kd_workspace_size_batch(n, count) bytes, as kd_decompose_batch.
+ * Errors: as kd_decompose_batch (argument checks first), KD_ERR_WORKSPACE for a null,
+ * unaligned or short staging buffer, KD_ERR_CUDA if a copy or launch fails to enqueue.
+ * The paper has no counterpart: this is the library's own end-to-end entry point. */
+typedef struct kd_matrix_host {
+  const void* w;
+  int64_t m;
+  int64_t ld;
+  uint64_t sign_seed;
+  uint32_t* codes_u;
+  uint32_t* codes_v;
+  float* centres_u;
+  float* centres_v;
+  float* coeffs;
+} kd_matrix_host;
+
+/* Device staging bytes kd_decompose_batch_host needs for these matrices (0 for an
+ * invalid count, size or enum). */
+size_t kd_staging_size_host(const kd_matrix_host* mats, int count, kd_dtype dtype, kd_layout layout, int64_t n);
+
+kd_status kd_decompose_batch_host(const kd_matrix_host* mats, int count, kd_dtype dtype, kd_layout layout,
+                                  int64_t n, int iters, int kmeans_iters, void* staging, size_t staging_bytes,
+                                  void* workspace, size_t ws_bytes, void* stream);
+
 /* y_j = P x_j for m vectors of length n, fp32, vector-major [m][n] contiguous
  * (Sec. 3.1: P z = IDCT(eps * DCT(z)); App. C uses the same operator on the rows
  * of the activations, XP).  x and y may alias; both 4-byte aligned

@@ -31,7 +31,7 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
-           "kd_read_status_static",
+           "kd_read_status_static", "kd_staging_size_host", "kd_decompose_batch_host",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
@@ -48,6 +48,13 @@ class KdRecMat(ctypes.Structure):
     _fields_ = [("codes_u", ctypes.c_void_p), ("codes_v", ctypes.c_void_p), ("centres_u", ctypes.c_void_p),
                 ("centres_v", ctypes.c_void_p), ("sign_seed", ctypes.c_uint64), ("w_hat", ctypes.c_void_p),
                 ("m", ctypes.c_int64), ("ld", ctypes.c_int64)]
+
+
+class KdMatrixHost(ctypes.Structure):
+    """Mirror of kd_matrix_host (include/kashin.h): every pointer is host memory."""
+    _fields_ = [("w", ctypes.c_void_p), ("m", ctypes.c_int64), ("ld", ctypes.c_int64),
+                ("sign_seed", ctypes.c_uint64), ("codes_u", ctypes.c_void_p), ("codes_v", ctypes.c_void_p),
+                ("centres_u", ctypes.c_void_p), ("centres_v", ctypes.c_void_p), ("coeffs", ctypes.c_void_p)]
 
 
 class KdMatrix(ctypes.Structure):
@@ -90,6 +97,11 @@ def _load() -> ctypes.CDLL:
     lib.kd_decompose_static.restype = c_int
     lib.kd_read_status_static.argtypes = [c_vp]
     lib.kd_read_status_static.restype = c_int
+    lib.kd_staging_size_host.argtypes = [c_vp, c_int, c_int, c_int, c_i64]
+    lib.kd_staging_size_host.restype = c_sz
+    lib.kd_decompose_batch_host.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp,
+                                            c_sz, c_vp]
+    lib.kd_decompose_batch_host.restype = c_int
     lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
     lib.kd_workspace_size_batch.restype = c_sz
     lib.kd_decompose_batch.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
@@ -201,6 +213,16 @@ def kd_decompose_static(w, dtype, layout, n, m, ld, sign_seed, iters, kmeans_ite
 
 def kd_read_status_static(stream) -> int:
     return lib.kd_read_status_static(stream)
+
+
+def kd_staging_size_host(mats, count, dtype, layout, n) -> int:
+    return int(lib.kd_staging_size_host(mats, count, dtype, layout, n))
+
+
+def kd_decompose_batch_host(mats, count, dtype, layout, n, iters, kmeans_iters, staging, staging_bytes, workspace,
+                            ws_bytes, stream) -> int:
+    return lib.kd_decompose_batch_host(mats, count, dtype, layout, n, iters, kmeans_iters, staging, staging_bytes,
+                                       workspace, ws_bytes, stream)
 
 
 def kd_dequantise(codes, centres, n, m, out_dtype, layout, out, ld, stream) -> int:
@@ -369,6 +391,63 @@ def decompose_batch(ws, iters: int, sign_seeds, layout: str = "rows", coeffs: bo
     if st != KD_OK:
         raise KashinError(st, "kd_decompose_batch")
     return res
+
+
+def _host_descriptors(ws, sign_seeds, layout, outs):
+    """kd_matrix_host array for host tensors ``ws`` and host outputs ``outs`` (one
+    Decomposed of CPU tensors per matrix)."""
+    if not 1 <= len(ws) <= KD_MAX_BATCH or len(sign_seeds) != len(ws) or len(outs) != len(ws):
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices with one seed and one output set each")
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    n = ws[0].shape[1] if lay == KD_VEC_ROWS else ws[0].shape[0]
+    arr = (KdMatrixHost * len(ws))()
+    for i, (w, o) in enumerate(zip(ws, outs)):
+        if w.is_cuda or w.dim() != 2 or w.stride(1) != 1 or w.dtype != ws[0].dtype:
+            raise ValueError("matrices must be 2-D host tensors of one dtype with unit inner stride")
+        m = w.shape[0] if lay == KD_VEC_ROWS else w.shape[1]
+        for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v, o.coeffs):
+            if t is not None and t.is_cuda:
+                raise ValueError("outputs must be host tensors")
+        arr[i] = KdMatrixHost(w.data_ptr(), m, w.stride(0), int(sign_seeds[i]) & ((1 << 64) - 1),
+                              _ptr(o.codes_u), _ptr(o.codes_v), _ptr(o.centres_u), _ptr(o.centres_v),
+                              _ptr(o.coeffs))
+    return arr, lay, n
+
+
+def host_outputs(m: int, n: int, coeffs: bool = False, pin: bool = True) -> Decomposed:
+    """Host (pinned) output tensors for one matrix of decompose_batch_host."""
+    torch = _torch()
+    def mk(shape, dt):
+        t = torch.empty(shape, dtype=dt)
+        return t.pin_memory() if pin else t
+    return Decomposed(codes_u=mk((m, (n + 15) // 16), torch.int32), codes_v=mk((m, (n + 15) // 16), torch.int32),
+                      centres_u=mk((m, 4), torch.float32), centres_v=mk((m, 4), torch.float32),
+                      coeffs=mk((m, 4), torch.float32) if coeffs else None, u=None, vhat=None, resid=None,
+                      trace=None)
+
+
+def staging_size_host(ws, layout: str = "rows", coeffs: bool = False) -> int:
+    """Device staging bytes decompose_batch_host needs for host matrices ``ws``."""
+    lay = KD_VEC_ROWS if layout == "rows" else KD_VEC_COLUMNS
+    n = ws[0].shape[1] if lay == KD_VEC_ROWS else ws[0].shape[0]
+    outs = [host_outputs(w.shape[0] if lay == KD_VEC_ROWS else w.shape[1], n, coeffs, pin=False) for w in ws]
+    arr, lay, n = _host_descriptors(ws, [0] * len(ws), layout, outs)
+    return kd_staging_size_host(ctypes.cast(arr, ctypes.c_void_p), len(ws), _dtype_code(ws[0].dtype), lay, n)
+
+
+def decompose_batch_host(ws, iters: int, sign_seeds, outs, staging, workspace: Workspace, layout: str = "rows",
+                         stream=None, kmeans_iters: int = 0):
+    """kd_decompose_batch_host: host matrices ``ws`` (pinned CPU tensors) in, host
+    outputs ``outs`` (from host_outputs) written once ``stream`` completes.  ``staging``
+    is a device uint8 tensor of at least staging_size_host(ws) bytes."""
+    arr, lay, n = _host_descriptors(ws, sign_seeds, layout, outs)
+    st = kd_decompose_batch_host(ctypes.cast(arr, ctypes.c_void_p), len(ws), _dtype_code(ws[0].dtype), lay, n,
+                                 int(iters), int(kmeans_iters), staging.data_ptr(),
+                                 staging.numel() * staging.element_size(), workspace.ptr, workspace.nbytes,
+                                 _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_decompose_batch_host")
+    return outs
 
 
 def read_status(workspace: Workspace, stream=None) -> int:

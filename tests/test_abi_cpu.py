@@ -273,3 +273,29 @@ def test_static_entry_checks_arguments_before_its_limit(kd):
     # valid arguments beyond the static array's limit
     assert st(16, 0, 0, 11008, 4, 11008, 0, 4, 0, 16, 16, 16, 16, null, null, null, null, null,
               null) == kd.KD_ERR_WORKSPACE
+
+
+def test_host_entry_validates_before_copying(kd):
+    """kd_decompose_batch_host refuses bad arguments and staging without a CUDA call."""
+    null = None
+    mats = (kd.KdMatrixHost * 2)()
+    mats[0] = kd.KdMatrixHost(16, 4, 256, 0, 16, 16, 16, 16, None)
+    mats[1] = kd.KdMatrixHost(16, 6, 256, 0, 16, 16, 16, 16, None)
+    arr = ctypes.cast(mats, ctypes.c_void_p)
+    f = kd.kd_decompose_batch_host
+    assert kd.kd_staging_size_host(arr, 2, kd.KD_F16, kd.KD_VEC_ROWS, 256) > 0
+    assert kd.kd_staging_size_host(arr, 0, kd.KD_F16, kd.KD_VEC_ROWS, 256) == 0
+    assert f(null, 1, 1, 0, 256, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert f(arr, 2, 9, 0, 256, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert f(arr, 2, 1, 0, 4094, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_UNSUPPORTED_N
+    assert f(arr, 2, 1, 0, 256, -1, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    # staging null, unaligned or short; workspace short
+    assert f(arr, 2, 1, 0, 256, 4, 0, null, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_WORKSPACE
+    assert f(arr, 2, 1, 0, 256, 4, 0, 128, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_WORKSPACE
+    assert f(arr, 2, 1, 0, 256, 4, 0, 256, 64, 16, 1 << 20, null) == kd.KD_ERR_WORKSPACE
+    assert f(arr, 2, 1, 0, 256, 4, 0, 256, 1 << 30, 16, 8, null) == kd.KD_ERR_WORKSPACE
+    # a matrix with m > 0 and a null output, then one whose ld is too small
+    mats[1] = kd.KdMatrixHost(16, 6, 256, 0, None, 16, 16, 16, None)
+    assert f(arr, 2, 1, 0, 256, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    mats[1] = kd.KdMatrixHost(16, 6, 255, 0, 16, 16, 16, 16, None)
+    assert f(arr, 2, 1, 0, 256, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
