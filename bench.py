@@ -539,6 +539,41 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
 
     ms_rec = timed(rec)
     ms_deq = timed(deq)
+
+    # the layer product straight from the 2-bit planes (kd_matmul_2bit, XP from
+    # kd_apply_p per matrix) against the dense fp16 product on the reconstructed W_hat
+    # (cuBLAS through torch.matmul), per batch of activation rows
+    dev = layer[0][1].device
+    wsp = {s.N: kd.Workspace(s.N, dev) for s, _ in layer}
+    folded = {}
+    for bsz in (1, 4, 16):
+        xs = {n: torch.randn((bsz, n), device=dev, dtype=torch.float32) for n in rec_groups}
+        xps = [torch.empty_like(xs[s.N]) for s, _ in decs]
+        ys = [torch.empty((bsz, s.M), device=dev, dtype=torch.float32) for s, _ in decs]
+        x16 = {n: x.half() for n, x in xs.items()}
+
+        def xp_all():
+            for (s, d), xp in zip(decs, xps):
+                kd.apply_p(xs[s.N], s.sign_seed, out=xp, workspace=wsp[s.N], stream=stream)
+
+        def prod_all():
+            for (s, d), xp, y in zip(decs, xps, ys):
+                kd.matmul_2bit(d, xs[s.N], xp, out=y, stream=stream)
+
+        def dense_all():
+            with torch.cuda.stream(stream):
+                for n, grp in rec_groups.items():
+                    for _, _, wh in grp:
+                        torch.matmul(x16[n], wh.T)
+
+        ms_xp, ms_prod, ms_dense = timed(xp_all, 6), timed(prod_all, 6), timed(dense_all, 6)
+        prod_bytes = sum(2 * s.M * ((s.N + 15) // 16) * 4 + 2 * s.M * 16 + 2 * bsz * s.N * 4 + bsz * s.M * 4
+                         for s, _ in layer)
+        folded[f"batch{bsz}"] = {
+            "ms_product": round(ms_prod, 4), "ms_xp": round(ms_xp, 4), "ms_total": round(ms_prod + ms_xp, 4),
+            "ms_dense_fp16": round(ms_dense, 4), "bound": "hbm",
+            "achieved": round(prod_bytes / (ms_prod / 1e3) / 1e9, 1), "peak": hbm_peak_gbs()[0], "unit": "GB/s",
+            "frac": round(prod_bytes / (ms_prod / 1e3) / 1e9 / hbm_peak_gbs()[0], 4)}
     params = sum(s.params for s, _ in layer)
     # one P (a DCT and an inverse DCT) per vector: 2 * 2 n log2 n flops, plus n adds
     import math
@@ -546,7 +581,7 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
     peak_alu = SM_COUNT * FP32_LANES_PER_SM * 2 * 2.070e9 / 1e12
     deq_bytes = 2 * params * (0.25 + 2)
     hbm, basis = hbm_peak_gbs()
-    del decs, planes_out, rec_groups
+    del planes_out
     return {
         "reconstruct": {"kernel": "reconstruct_kernel (codes -> fp16 W_hat, one kd_reconstruct_batch per vector "
                                   "length)",
@@ -560,6 +595,11 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
                        "achieved": round(deq_bytes / (ms_deq / 1e3) / 1e9, 1), "peak": hbm, "unit": "GB/s",
                        "frac": round(deq_bytes / (ms_deq / 1e3) / 1e9 / hbm, 4), "peak_basis": basis,
                        "algorithmic_bytes_per_param": 4.5},
+        "matmul_2bit": {"kernel": "fold_kernel (Y = X U_q^T + XP V_q^T from the 2-bit planes, one launch per "
+                                  "matrix and group of up to 4 rows; XP by kd_apply_p per matrix) against "
+                                  "torch.matmul fp16 on W_hat (cuBLAS), whole layer",
+                        "algorithmic_bytes": "codes 0.5 B per weight + centres + x, XP, y", "peak_basis": basis,
+                        **folded},
     }
 
 

@@ -325,6 +325,25 @@ kd_status kd_dequantise_batch(const kd_plane* planes, int count, int64_t n, kd_d
  * Used as the measured denominator of the transform kernels' ALU roofline. */
 kd_status kd_measure_fp32_peak(double* tflops, void* stream);
 
+/* The layer product straight from the 2-bit planes (App. C: X W = X U_q + (X P) V_q =
+ * [X | XP] [U_q; V_q], evaluated without expanding U_q or V_q):
+ *   y[r*ldy + j] = sum_i centres_u[j][code_u(j,i)] x[r*ldx + i]
+ *                + sum_i centres_v[j][code_v(j,i)] xp[r*ldx + i],   r < batch, j < m,
+ * i.e. Y = X W_hat^T for the m vectors (output channels) of W_hat = U_q + P V_q.
+ *   codes_u, codes_v   device, m x ceil(n/16) uint32, 4-byte aligned (kd_decompose's).
+ *   centres_u, _v      device, m x 4 fp32 ascending, 16-byte aligned.
+ *   x                  device fp32, batch rows of n inputs, row r at x + r*ldx (ldx >= n).
+ *   xp                 device fp32, the same rows times P (kd_apply_p with the matrix's
+ *                      sign seed on the rows of X), same layout and ldx.
+ *   y                  device fp32, batch rows of m outputs, row r at y + r*ldy (ldy >= m).
+ * Every code word is read once per group of up to four batch rows; accumulation is
+ * fp32 in a fixed order (deterministic).  Errors: KD_ERR_INVALID_ARG (sizes, null or
+ * unaligned pointers when m > 0 and batch > 0), KD_ERR_CUDA (launch).  m == 0 or
+ * batch == 0 enqueues nothing. */
+kd_status kd_matmul_2bit(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
+                         const float* centres_v, int64_t n, int64_t m, const float* x, const float* xp,
+                         int64_t batch, int64_t ldx, float* y, int64_t ldy, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:
  * the weights are rotated by a randomized Hadamard transform before the

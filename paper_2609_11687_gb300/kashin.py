@@ -32,6 +32,7 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_read_status_static", "kd_staging_size_host", "kd_decompose_batch_host",
+           "kd_matmul_2bit",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
@@ -102,6 +103,8 @@ def _load() -> ctypes.CDLL:
     lib.kd_decompose_batch_host.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp,
                                             c_sz, c_vp]
     lib.kd_decompose_batch_host.restype = c_int
+    lib.kd_matmul_2bit.argtypes = [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_vp, c_vp, c_i64, c_i64, c_vp, c_i64, c_vp]
+    lib.kd_matmul_2bit.restype = c_int
     lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
     lib.kd_workspace_size_batch.restype = c_sz
     lib.kd_decompose_batch.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
@@ -391,6 +394,32 @@ def decompose_batch(ws, iters: int, sign_seeds, layout: str = "rows", coeffs: bo
     if st != KD_OK:
         raise KashinError(st, "kd_decompose_batch")
     return res
+
+
+def kd_matmul_2bit(codes_u, codes_v, centres_u, centres_v, n, m, x, xp, batch, ldx, y, ldy, stream) -> int:
+    return lib.kd_matmul_2bit(codes_u, codes_v, centres_u, centres_v, n, m, x, xp, batch, ldx, y, ldy, stream)
+
+
+def matmul_2bit(dec: "Decomposed", x, xp, out=None, stream=None):
+    """``Y = X W_hat^T`` from the code planes (App. C): ``x`` and ``xp`` (= apply_p of the
+    rows of x with the matrix's sign seed) are fp32 CUDA tensors (batch, n); returns
+    (batch, m) fp32."""
+    torch = _torch()
+    m, words = dec.codes_u.shape
+    if x.dim() != 2 or x.dtype != torch.float32 or xp.shape != x.shape or xp.dtype != x.dtype:
+        raise ValueError("x and xp must be fp32 (batch, n) tensors of one shape")
+    if x.stride(1) != 1 or xp.stride(1) != 1 or x.stride(0) != xp.stride(0):
+        raise ValueError("x and xp need unit inner stride and equal row strides")
+    b, n = x.shape
+    if (n + 15) // 16 != words:
+        raise ValueError("x does not match the code planes' vector length")
+    y = out if out is not None else torch.empty((b, m), dtype=torch.float32, device=x.device)
+    st = kd_matmul_2bit(dec.codes_u.data_ptr(), dec.codes_v.data_ptr(), dec.centres_u.data_ptr(),
+                        dec.centres_v.data_ptr(), n, m, x.data_ptr(), xp.data_ptr(), b, x.stride(0), y.data_ptr(),
+                        y.stride(0), _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_matmul_2bit")
+    return y
 
 
 def _host_descriptors(ws, sign_seeds, layout, outs):

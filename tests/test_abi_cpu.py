@@ -299,3 +299,18 @@ def test_host_entry_validates_before_copying(kd):
     assert f(arr, 2, 1, 0, 256, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     mats[1] = kd.KdMatrixHost(16, 6, 255, 0, 16, 16, 16, 16, None)
     assert f(arr, 2, 1, 0, 256, 4, 0, 256, 1 << 30, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+
+
+def test_matmul_2bit_validation(kd):
+    """kd_matmul_2bit refuses bad sizes, null and unaligned pointers without a CUDA call."""
+    f = kd.kd_matmul_2bit
+    null = None
+    assert f(16, 16, 16, 16, 0, 4, 16, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG       # n = 0
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, 1, 255, 16, 4, null) == kd.KD_ERR_INVALID_ARG     # ldx < n
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, 1, 256, 16, 3, null) == kd.KD_ERR_INVALID_ARG     # ldy < m
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, -1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG    # batch < 0
+    assert f(16, null, 16, 16, 256, 4, 16, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG
+    assert f(16, 16, 8, 16, 256, 4, 16, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG      # centres 8-aligned
+    assert f(16, 16, 16, 16, 256, 4, 18, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG     # x unaligned
+    assert f(null, null, null, null, 256, 0, null, null, 1, 256, null, 0, null) == kd.KD_OK    # m == 0
+    assert f(null, null, null, null, 256, 4, null, null, 0, 256, null, 4, null) == kd.KD_OK    # batch == 0

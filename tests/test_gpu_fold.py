@@ -1,0 +1,102 @@
+"""kd_matmul_2bit: the layer product straight from the 2-bit planes (App. C,
+Y = X U_q^T + (X P) V_q^T), against the fp64 oracle.
+
+The oracle expands the device's codes and centres itself (oracle.dequantise) and
+applies its own dense P to the rows of X, in fp64; the device runs kd_apply_p for XP
+and the product kernel.  Both sides use the device's codes and centres: the product
+is what is checked here (which codes a decomposition picks is the decomposition's
+parity, checked elsewhere).  Tolerance: 1e-5 of max |Y| per batch row."""
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import kashin_oracle as ko
+from paper_2609_11687_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+TOL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def kd():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2609_11687_gb300 import build
+    build.build()
+    from paper_2609_11687_gb300 import kashin
+    return kashin
+
+
+_P = {}
+
+
+def _oracle_y(kd, dec, n, seed, x64):
+    """fp64: X U_q^T + (X P) V_q^T from the device's codes and centres."""
+    cu = ko.dequantise(kd.unpack_codes(dec.codes_u, n).T, dec.centres_u.double().cpu().numpy())  # (n, m)
+    cv = ko.dequantise(kd.unpack_codes(dec.codes_v, n).T, dec.centres_v.double().cpu().numpy())
+    if (n, seed) not in _P:
+        _P[(n, seed)] = ko.POperator(n, ko.sign_mask(seed, n))
+    xp = _P[(n, seed)](x64.T).T                                              # rows of X times P
+    return x64 @ cu + xp @ cv
+
+
+def _run(kd, w, seed, batch, iters=16, gen_seed=0):
+    m, n = w.shape
+    dec = kd.decompose(w, iters, seed)
+    g = torch.Generator(device="cuda").manual_seed(gen_seed)
+    x = torch.randn((batch, n), generator=g, device="cuda", dtype=torch.float32)
+    xp = kd.apply_p(x, seed)
+    y = kd.matmul_2bit(dec, x, xp)
+    torch.cuda.synchronize()
+    y_ora = _oracle_y(kd, dec, n, seed, x.double().cpu().numpy())
+    err = np.abs(y.double().cpu().numpy() - y_ora).max(axis=1)
+    scale = np.abs(y_ora).max(axis=1)
+    assert (err <= TOL * scale).all(), (err / scale).max()
+    return dec, x, xp, y
+
+
+@pytest.mark.parametrize("name", ["L0.q", "L0.gate", "L0.down"])
+@pytest.mark.parametrize("batch", [1, 3, 4])
+def test_matmul_2bit_7b_shapes(kd, name, batch):
+    """The 7B layer's 4096 x 4096, 4096 x 11008 and 11008 x 4096 matrices, whole."""
+    spec = {s.name: s for s in synth.config3()}[name]
+    w = synth.generate(spec, device="cuda")
+    _run(kd, w, spec.sign_seed, batch, gen_seed=batch)
+
+
+@pytest.mark.parametrize("n,m,batch", [(768, 37, 6), (1000, 19, 5), (256, 1, 2), (16, 9, 1)])
+def test_matmul_2bit_ragged(kd, n, m, batch):
+    """Channel counts that leave a partial tile, a length with a partial last code word
+    (run-time-length path), a single channel, the shortest length; batch chunks 4+2,
+    4+1, 2, 1."""
+    g = torch.Generator(device="cuda").manual_seed(n + m)
+    w = (torch.randn((m, n), generator=g, device="cuda") * 0.02).half()
+    _run(kd, w, 7, batch)
+
+
+def test_matmul_2bit_matches_reconstructed_weight(kd):
+    """The folded product equals X W_hat^T with W_hat from kd_reconstruct (fp32, the
+    load-time path), to fp32 rounding."""
+    g = torch.Generator(device="cuda").manual_seed(2)
+    w = (torch.randn((300, 4096), generator=g, device="cuda") * 0.02).half()
+    dec, x, xp, y = _run(kd, w, 11, 2)
+    wh = kd.reconstruct(dec, 4096, 11, dtype=torch.float32)
+    ref = x.double() @ wh.double().T
+    torch.cuda.synchronize()
+    err = (y.double() - ref).abs().amax(dim=1)
+    assert (err <= TOL * ref.abs().amax(dim=1)).all()
+
+
+def test_matmul_2bit_deterministic_and_empty(kd):
+    g = torch.Generator(device="cuda").manual_seed(3)
+    w = (torch.randn((64, 512), generator=g, device="cuda") * 0.02).half()
+    dec = kd.decompose(w, 8, 4)
+    x = torch.randn((3, 512), generator=g, device="cuda")
+    xp = kd.apply_p(x, 4)
+    a = kd.matmul_2bit(dec, x, xp)
+    b = kd.matmul_2bit(dec, x, xp)
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
+    e = kd.matmul_2bit(dec, x[:0], xp[:0])
+    assert e.shape == (0, 64)
