@@ -540,25 +540,29 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
     ms_rec = timed(rec)
     ms_deq = timed(deq)
 
-    # the layer product straight from the 2-bit planes (kd_matmul_2bit, XP from
-    # kd_apply_p per matrix) against the dense fp16 product on the reconstructed W_hat
-    # (cuBLAS through torch.matmul), per batch of activation rows
+    # the layer product straight from the 2-bit planes (one kd_matmul_2bit_batch for
+    # the layer, XP from one kd_apply_p_batch per vector length) against the dense fp16
+    # product on the reconstructed W_hat (cuBLAS through torch.matmul), per batch of
+    # activation rows
     dev = layer[0][1].device
-    wsp = {s.N: kd.Workspace(s.N, dev) for s, _ in layer}
+    by_n = {}
+    for k, (s_, _) in enumerate(decs):
+        by_n.setdefault(s_.N, []).append(k)
+    wsp = {n: kd.Workspace(n, dev, count=len(ix)) for n, ix in by_n.items()}
     folded = {}
     for bsz in (1, 4, 16):
         xs = {n: torch.randn((bsz, n), device=dev, dtype=torch.float32) for n in rec_groups}
-        xps = [torch.empty_like(xs[s.N]) for s, _ in decs]
-        ys = [torch.empty((bsz, s.M), device=dev, dtype=torch.float32) for s, _ in decs]
+        xps = [torch.empty_like(xs[s_.N]) for s_, _ in decs]
+        ys = [torch.empty((bsz, s_.M), device=dev, dtype=torch.float32) for s_, _ in decs]
         x16 = {n: x.half() for n, x in xs.items()}
 
         def xp_all():
-            for (s, d), xp in zip(decs, xps):
-                kd.apply_p(xs[s.N], s.sign_seed, out=xp, workspace=wsp[s.N], stream=stream)
+            for n, ix in by_n.items():
+                kd.apply_p_batch([xs[n]] * len(ix), [decs[k][0].sign_seed for k in ix], outs=[xps[k] for k in ix],
+                                 workspace=wsp[n], stream=stream)
 
         def prod_all():
-            for (s, d), xp, y in zip(decs, xps, ys):
-                kd.matmul_2bit(d, xs[s.N], xp, out=y, stream=stream)
+            kd.matmul_2bit_batch([d for _, d in decs], [xs[s_.N] for s_, _ in decs], xps, outs=ys, stream=stream)
 
         def dense_all():
             with torch.cuda.stream(stream):
@@ -595,9 +599,10 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
                        "achieved": round(deq_bytes / (ms_deq / 1e3) / 1e9, 1), "peak": hbm, "unit": "GB/s",
                        "frac": round(deq_bytes / (ms_deq / 1e3) / 1e9 / hbm, 4), "peak_basis": basis,
                        "algorithmic_bytes_per_param": 4.5},
-        "matmul_2bit": {"kernel": "fold_kernel (Y = X U_q^T + XP V_q^T from the 2-bit planes, one launch per "
-                                  "matrix and group of up to 4 rows; XP by kd_apply_p per matrix) against "
-                                  "torch.matmul fp16 on W_hat (cuBLAS), whole layer",
+        "matmul_2bit": {"kernel": "fold_kernel (Y = X U_q^T + XP V_q^T from the 2-bit planes: one "
+                                  "kd_matmul_2bit_batch per layer and group of up to 2 rows; XP by one "
+                                  "kd_apply_p_batch per vector length) against torch.matmul fp16 on W_hat "
+                                  "(cuBLAS, one call per matrix), whole layer",
                         "algorithmic_bytes": "codes 0.5 B per weight + centres + x, XP, y", "peak_basis": basis,
                         **folded},
     }

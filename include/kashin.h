@@ -247,6 +247,25 @@ kd_status kd_decompose_batch_host(const kd_matrix_host* mats, int count, kd_dtyp
 kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t sign_seed,
                      void* workspace, size_t ws_bytes, void* stream);
 
+/* kd_apply_p for several matrices of one vector length n in one launch (the XP of a
+ * layer's products, App. C), each with its own rows, output and sign seed:
+ *   mats       HOST array of 1 <= count <= KD_MAX_BATCH descriptors, read during the call;
+ *              y_j = P x_j for the m rows of x ([m][n] fp32 contiguous), x and y may alias.
+ *   workspace  16-byte aligned, ws_bytes >= kd_workspace_size_batch(n, count).
+ * Results equal kd_apply_p's per matrix, bit for bit.  Lengths above 8192 and the
+ * run-time-length path run one launch per matrix, in order, on the same stream and
+ * workspace.  Errors as kd_apply_p (the first invalid matrix's), and
+ * KD_ERR_INVALID_ARG for a bad count or a null array. */
+typedef struct kd_pmat {
+  const float* x;
+  float* y;
+  int64_t m;
+  uint64_t sign_seed;
+} kd_pmat;
+
+kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
+                           void* stream);
+
 /* Dense re-materialisation W_hat = U_q + P V_q (App. C): vector j of w_hat is
  * centres_u[j][code_u] + P(centres_v[j][code_v]).  Inputs as produced by
  * kd_decompose (centres 16-byte aligned, codes 4-byte aligned, KD_ERR_INVALID_ARG
@@ -336,13 +355,35 @@ kd_status kd_measure_fp32_peak(double* tflops, void* stream);
  *   xp                 device fp32, the same rows times P (kd_apply_p with the matrix's
  *                      sign seed on the rows of X), same layout and ldx.
  *   y                  device fp32, batch rows of m outputs, row r at y + r*ldy (ldy >= m).
- * Every code word is read once per group of up to four batch rows; accumulation is
+ * Every code word is read once per group of up to two batch rows; accumulation is
  * fp32 in a fixed order (deterministic).  Errors: KD_ERR_INVALID_ARG (sizes, null or
  * unaligned pointers when m > 0 and batch > 0), KD_ERR_CUDA (launch).  m == 0 or
  * batch == 0 enqueues nothing. */
 kd_status kd_matmul_2bit(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
                          const float* centres_v, int64_t n, int64_t m, const float* x, const float* xp,
                          int64_t batch, int64_t ldx, float* y, int64_t ldy, void* stream);
+
+/* kd_matmul_2bit for several matrices in one launch (a layer's products for one batch
+ * of activations): each descriptor as kd_matmul_2bit's arguments, each matrix with its
+ * own n, m, inputs and output.  mats is a HOST array of 1 <= count <= KD_MAX_BATCH
+ * descriptors read during the call.  Results equal kd_matmul_2bit's per matrix, bit for
+ * bit.  Errors as kd_matmul_2bit (the first invalid matrix's), and KD_ERR_INVALID_ARG
+ * for a bad count or a null array. */
+typedef struct kd_fold_mat {
+  const uint32_t* codes_u;
+  const uint32_t* codes_v;
+  const float* centres_u;
+  const float* centres_v;
+  const float* x;
+  const float* xp;
+  float* y;
+  int64_t n;
+  int64_t m;
+  int64_t ldx;
+  int64_t ldy;
+} kd_fold_mat;
+
+kd_status kd_matmul_2bit_batch(const kd_fold_mat* mats, int count, int64_t batch, void* stream);
 
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:

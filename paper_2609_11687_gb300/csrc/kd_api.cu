@@ -374,7 +374,60 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
   const int grid = grid_for(p.npairs, ops->q, per * sms);
-  return ops->apply(p, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+  return ops->apply(p, nullptr, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  if (!mats || count < 1 || count > KD_MAX_BATCH || n <= 0) return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  ApplyBatch ab;
+  ab.count = count;
+  int64_t npairs = 0;
+  for (int i = 0; i < count; ++i) {
+    const kd_pmat& a = mats[i];
+    if (a.m < 0) return KD_ERR_INVALID_ARG;
+    if (a.m > 0 && (!a.x || !a.y)) return KD_ERR_INVALID_ARG;
+    if (!aligned_to(a.x, 4) || !aligned_to(a.y, 4)) return KD_ERR_INVALID_ARG;
+    ab.mat[i].x = a.x;
+    ab.mat[i].y = a.y;
+    ab.mat[i].m = a.m;
+    ab.mat[i].pair0 = npairs;
+    npairs += (a.m + 1) / 2;
+  }
+  WsLayout L;
+  if (!layout_of(ops, &L, count)) return KD_ERR_CUDA;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (!ops->batch) {
+    // long vectors and the run-time-length path: one launch per matrix, in stream order
+    for (int i = 0; i < count; ++i) {
+      const kd_status sti = kd_apply_p(mats[i].x, mats[i].y, n, mats[i].m, mats[i].sign_seed, workspace, ws_bytes,
+                                       stream);
+      if (sti != KD_OK) return sti;
+    }
+    return KD_OK;
+  }
+  uint64_t seeds[KD_MAX_BATCH];
+  for (int i = 0; i < count; ++i) seeds[i] = mats[i].sign_seed;
+  kd_status st = setup_batch(ops, L, workspace, seeds, count, n, s);
+  if (st != KD_OK || npairs == 0) return st;
+  char* b = static_cast<char*>(workspace);
+  ApplyParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.n = n;
+  p.m = mats[0].m;
+  p.x = mats[0].x;
+  p.y = mats[0].y;
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.npairs = npairs;
+  const int per = ops->ctas_per_sm(1, n);
+  const int sms = sm_count();
+  if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
+  const int grid = grid_for(p.npairs, ops->q, per * sms);
+  return ops->apply(p, &ab, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
 kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,

@@ -618,7 +618,7 @@ cudaError_t gen_decompose(const DecParams& p, const BatchParams* bp, int grid, c
   return cudaGetLastError();
 }
 
-cudaError_t gen_apply_launch(const ApplyParams& p, int grid, cudaStream_t s) {
+cudaError_t gen_apply_launch(const ApplyParams& p, const ApplyBatch*, int grid, cudaStream_t s) {
   GenPlan g;
   if (!gen_plan(p.n, &g)) return cudaErrorInvalidValue;
   const size_t smem = gen_smem(p.n);

@@ -697,8 +697,22 @@ struct ApplyParams {
   int64_t npairs;
 };
 
+// Several matrices of one vector length in one kd_apply_p launch (kd_apply_p_batch):
+// matrix i owns the global pairs [pair0, pair0 + ceil(m / 2)) and the sign bits at
+// eps + i * ceil(n / 32).
+struct ApplyMat {
+  const float* x;
+  float* y;
+  int64_t m, pair0;
+};
+struct ApplyBatch {
+  int count;  // 0: the single matrix of ApplyParams
+  ApplyMat mat[kMaxBatch];
+};
+
 template <class PL>
-__global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyParams p) {
+__global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyParams p,
+                                                                        const __grid_constant__ ApplyBatch ab) {
   constexpr int N = PL::N;
   constexpr int T = PL::T;
   constexpr int E = PL::E;
@@ -709,17 +723,31 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyPar
   float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
   Xform<PL, false> xf;  // scalar roots: no registers to spare for constant pairs
   xf.init(buf, tw, p.eps, lt);
+  int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
   for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
     const int64_t pair = base + team;
     const bool active = pair < p.npairs;
-    const int64_t pr = active ? pair : base;
+    int64_t pr = active ? pair : base;
+    int mi = 0;
+    const bool batched = PL::BATCH && ab.count > 0;
+    if (batched) {
+      while (mi + 1 < ab.count && pr >= ab.mat[mi + 1].pair0) ++mi;
+      pr -= ab.mat[mi].pair0;
+      if (mi != cur_mat) {  // uniform per team: Q == 1 whenever T > 32
+        xf.set_eps(p.eps + (int64_t)mi * ((N + 31) / 32));
+        cur_mat = mi;
+      }
+    }
+    const float* x = batched ? ab.mat[mi].x : p.x;
+    float* y = batched ? ab.mat[mi].y : p.y;
+    const int64_t m_in = batched ? ab.mat[mi].m : p.m;
     const int64_t colA = 2 * pr;
-    const bool hasB = (colA + 1) < p.m;
+    const bool hasB = (colA + 1) < m_in;
     float2 v[E];
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
-      v[j] = make_float2(__ldg(&p.x[colA * N + nat]), hasB ? __ldg(&p.x[(colA + 1) * N + nat]) : 0.f);
+      v[j] = make_float2(__ldg(&x[colA * N + nat]), hasB ? __ldg(&x[(colA + 1) * N + nat]) : 0.f);
     }
     team_sync<PL>();  // x and y may alias: all loads of this pair precede any store
     xf.apply(v);
@@ -727,8 +755,8 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyPar
 #pragma unroll
       for (int j = 0; j < E; ++j) {
         const int nat = nat_of<N>(lt + j * T);
-        p.y[colA * N + nat] = v[j].x;
-        if (hasB) p.y[(colA + 1) * N + nat] = v[j].y;
+        y[colA * N + nat] = v[j].x;
+        if (hasB) y[(colA + 1) * N + nat] = v[j].y;
       }
     }
     team_sync<PL>();

@@ -48,11 +48,16 @@ struct Ops {
     }
     return cudaGetLastError();
   }
-  static cudaError_t apply(const ApplyParams& p, int grid, cudaStream_t s) {
+  static cudaError_t apply(const ApplyParams& p, const ApplyBatch* ab, int grid, cudaStream_t s) {
     auto k = apply_p_kernel<PL>;
     cudaError_t e = prepare(k, PL::SMEM);
     if (e != cudaSuccess) return e;
-    k<<<grid, PL::THREADS, PL::SMEM, s>>>(p);
+    if (ab) {
+      k<<<grid, PL::THREADS, PL::SMEM, s>>>(p, *ab);
+    } else {
+      ApplyBatch none{};
+      k<<<grid, PL::THREADS, PL::SMEM, s>>>(p, none);
+    }
     return cudaGetLastError();
   }
   static cudaError_t setup(float2* twt, uint32_t* eps, uint32_t* status, uint64_t seed, int64_t, cudaStream_t s) {

@@ -10,6 +10,7 @@ namespace kd {
 struct DecParams;
 struct BatchParams;
 struct ApplyParams;
+struct ApplyBatch;
 struct RecParams;
 struct RecBatch;
 
@@ -25,7 +26,8 @@ struct PlanOps {
   int (*ctas_per_sm)(int which, int64_t n);  // which: 0 decompose, 1 apply, 2 reconstruct
   // bp: the matrices of a batched launch, or nullptr for DecParams' single matrix
   cudaError_t (*decompose)(const DecParams&, const BatchParams* bp, int grid, cudaStream_t);
-  cudaError_t (*apply)(const ApplyParams&, int grid, cudaStream_t);
+  // ab: the matrices of a batched launch (plans with batch only), or nullptr
+  cudaError_t (*apply)(const ApplyParams&, const ApplyBatch* ab, int grid, cudaStream_t);
   // rb: the matrices of a batched launch, or nullptr for RecParams' single matrix
   cudaError_t (*reconstruct)(const RecParams&, const RecBatch* rb, int grid, cudaStream_t);
   // tables for one call of vector length n: twiddles (float2[twn]), sign bits, cleared status word

@@ -32,7 +32,7 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_read_status_static", "kd_staging_size_host", "kd_decompose_batch_host",
-           "kd_matmul_2bit",
+           "kd_matmul_2bit", "kd_matmul_2bit_batch", "kd_apply_p_batch",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
@@ -49,6 +49,19 @@ class KdRecMat(ctypes.Structure):
     _fields_ = [("codes_u", ctypes.c_void_p), ("codes_v", ctypes.c_void_p), ("centres_u", ctypes.c_void_p),
                 ("centres_v", ctypes.c_void_p), ("sign_seed", ctypes.c_uint64), ("w_hat", ctypes.c_void_p),
                 ("m", ctypes.c_int64), ("ld", ctypes.c_int64)]
+
+
+class KdPMat(ctypes.Structure):
+    """Mirror of kd_pmat (include/kashin.h): rows x -> y = P x with one sign seed."""
+    _fields_ = [("x", ctypes.c_void_p), ("y", ctypes.c_void_p), ("m", ctypes.c_int64), ("sign_seed", ctypes.c_uint64)]
+
+
+class KdFoldMat(ctypes.Structure):
+    """Mirror of kd_fold_mat (include/kashin.h): one matrix of kd_matmul_2bit_batch."""
+    _fields_ = [("codes_u", ctypes.c_void_p), ("codes_v", ctypes.c_void_p), ("centres_u", ctypes.c_void_p),
+                ("centres_v", ctypes.c_void_p), ("x", ctypes.c_void_p), ("xp", ctypes.c_void_p),
+                ("y", ctypes.c_void_p), ("n", ctypes.c_int64), ("m", ctypes.c_int64), ("ldx", ctypes.c_int64),
+                ("ldy", ctypes.c_int64)]
 
 
 class KdMatrixHost(ctypes.Structure):
@@ -105,6 +118,10 @@ def _load() -> ctypes.CDLL:
     lib.kd_decompose_batch_host.restype = c_int
     lib.kd_matmul_2bit.argtypes = [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_vp, c_vp, c_i64, c_i64, c_vp, c_i64, c_vp]
     lib.kd_matmul_2bit.restype = c_int
+    lib.kd_matmul_2bit_batch.argtypes = [c_vp, c_int, c_i64, c_vp]
+    lib.kd_matmul_2bit_batch.restype = c_int
+    lib.kd_apply_p_batch.argtypes = [c_vp, c_int, c_i64, c_vp, c_sz, c_vp]
+    lib.kd_apply_p_batch.restype = c_int
     lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
     lib.kd_workspace_size_batch.restype = c_sz
     lib.kd_decompose_batch.argtypes = [c_vp, c_int, c_int, c_int, c_i64, c_int, c_int, c_vp, c_sz, c_vp]
@@ -420,6 +437,63 @@ def matmul_2bit(dec: "Decomposed", x, xp, out=None, stream=None):
     if st != KD_OK:
         raise KashinError(st, "kd_matmul_2bit")
     return y
+
+
+def kd_matmul_2bit_batch(mats, count, batch, stream) -> int:
+    return lib.kd_matmul_2bit_batch(mats, count, batch, stream)
+
+
+def kd_apply_p_batch(mats, count, n, workspace, ws_bytes, stream) -> int:
+    return lib.kd_apply_p_batch(mats, count, n, workspace, ws_bytes, stream)
+
+
+def matmul_2bit_batch(decs, xs, xps, outs=None, stream=None):
+    """kd_matmul_2bit_batch: ``Y_i = X_i W_hat_i^T`` for several matrices in one launch
+    (``decs`` Decomposed, ``xs``/``xps`` fp32 (batch, n_i) CUDA tensors, one batch size)."""
+    torch = _torch()
+    if not 1 <= len(decs) <= KD_MAX_BATCH or len(xs) != len(decs) or len(xps) != len(decs):
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices with one x and one xp each")
+    b = xs[0].shape[0]
+    arr = (KdFoldMat * len(decs))()
+    res = []
+    for i, (d, x, xp) in enumerate(zip(decs, xs, xps)):
+        m, words = d.codes_u.shape
+        if x.dim() != 2 or x.shape[0] != b or x.dtype != torch.float32 or xp.shape != x.shape \
+                or xp.dtype != x.dtype or x.stride(1) != 1 or xp.stride(1) != 1 or x.stride(0) != xp.stride(0):
+            raise ValueError("x and xp must be fp32 (batch, n) tensors of one shape, unit inner stride")
+        n = x.shape[1]
+        if (n + 15) // 16 != words:
+            raise ValueError("x does not match the code planes' vector length")
+        y = outs[i] if outs is not None else torch.empty((b, m), dtype=torch.float32, device=x.device)
+        arr[i] = KdFoldMat(d.codes_u.data_ptr(), d.codes_v.data_ptr(), d.centres_u.data_ptr(), d.centres_v.data_ptr(),
+                           x.data_ptr(), xp.data_ptr(), y.data_ptr(), n, m, x.stride(0), y.stride(0))
+        res.append(y)
+    st = kd_matmul_2bit_batch(ctypes.cast(arr, ctypes.c_void_p), len(decs), b, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_matmul_2bit_batch")
+    return res
+
+
+def apply_p_batch(xs, sign_seeds, outs=None, workspace: Optional[Workspace] = None, stream=None):
+    """kd_apply_p_batch: ``y = P x`` for the rows of several fp32 (m_i, n) tensors, each
+    with its own sign seed, in one launch."""
+    torch = _torch()
+    if not 1 <= len(xs) <= KD_MAX_BATCH or len(sign_seeds) != len(xs):
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices with one seed each")
+    n = xs[0].shape[1]
+    arr = (KdPMat * len(xs))()
+    res = []
+    for i, x in enumerate(xs):
+        if x.dtype != torch.float32 or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != n:
+            raise ValueError("inputs must be contiguous fp32 (m, n) CUDA tensors of one n")
+        y = outs[i] if outs is not None else torch.empty_like(x)
+        arr[i] = KdPMat(x.data_ptr(), y.data_ptr(), x.shape[0], int(sign_seeds[i]) & ((1 << 64) - 1))
+        res.append(y)
+    ws = workspace if workspace is not None else Workspace(n, xs[0].device, count=len(xs))
+    st = kd_apply_p_batch(ctypes.cast(arr, ctypes.c_void_p), len(xs), n, ws.ptr, ws.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_apply_p_batch")
+    return res
 
 
 def _host_descriptors(ws, sign_seeds, layout, outs):

@@ -314,3 +314,23 @@ def test_matmul_2bit_validation(kd):
     assert f(16, 16, 16, 16, 256, 4, 18, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG     # x unaligned
     assert f(null, null, null, null, 256, 0, null, null, 1, 256, null, 0, null) == kd.KD_OK    # m == 0
     assert f(null, null, null, null, 256, 4, null, null, 0, 256, null, 4, null) == kd.KD_OK    # batch == 0
+
+
+def test_batched_product_and_transform_validation(kd):
+    null = None
+    mats = (kd.KdFoldMat * 2)()
+    mats[0] = kd.KdFoldMat(16, 16, 16, 16, 16, 16, 16, 256, 4, 256, 4)
+    mats[1] = kd.KdFoldMat(16, 16, 8, 16, 16, 16, 16, 256, 4, 256, 4)      # centres not 16-byte aligned
+    arr = ctypes.cast(mats, ctypes.c_void_p)
+    assert kd.kd_matmul_2bit_batch(null, 1, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_batch(arr, 0, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_batch(arr, 2, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_batch(arr, 1, -1, null) == kd.KD_ERR_INVALID_ARG
+    pm = (kd.KdPMat * 2)()
+    pm[0] = kd.KdPMat(16, 16, 4, 1)
+    pm[1] = kd.KdPMat(16, 6, 4, 2)                                         # y not 4-byte aligned
+    parr = ctypes.cast(pm, ctypes.c_void_p)
+    assert kd.kd_apply_p_batch(null, 1, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_apply_p_batch(parr, 1, 4094, 16, 1 << 20, null) == kd.KD_ERR_UNSUPPORTED_N
+    assert kd.kd_apply_p_batch(parr, 2, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_apply_p_batch(parr, 1, 256, null, 1 << 20, null) == kd.KD_ERR_WORKSPACE

@@ -100,3 +100,22 @@ def test_matmul_2bit_deterministic_and_empty(kd):
     assert torch.equal(a, b)
     e = kd.matmul_2bit(dec, x[:0], xp[:0])
     assert e.shape == (0, 64)
+
+
+def test_batched_calls_equal_single_calls(kd):
+    """kd_apply_p_batch and kd_matmul_2bit_batch over a layer-like set of matrices (two
+    vector lengths, ragged counts) reproduce the single calls bit for bit."""
+    g = torch.Generator(device="cuda").manual_seed(9)
+    shapes = [(37, 768, 3), (64, 768, 4), (5, 768, 5), (21, 11008, 6)]
+    decs, xs, xps = [], [], []
+    for m, n, seed in shapes:
+        w = (torch.randn((m, n), generator=g, device="cuda") * 0.02).half()
+        decs.append(kd.decompose(w, 4, seed))
+        xs.append(torch.randn((3, n), generator=g, device="cuda"))
+    xps = kd.apply_p_batch(xs[:3], [3, 4, 5]) + kd.apply_p_batch(xs[3:], [6])
+    ys = kd.matmul_2bit_batch(decs, xs, xps)
+    for (m, n, seed), d, x, xp, y in zip(shapes, decs, xs, xps, ys):
+        xp1 = kd.apply_p(x, seed)
+        y1 = kd.matmul_2bit(d, x, xp1)
+        torch.cuda.synchronize()
+        assert torch.equal(xp, xp1) and torch.equal(y, y1)
