@@ -153,6 +153,12 @@ bool outputs_aligned(const void* w, int dtype, const void* codes_u, const void* 
 }
 bool valid_layout(int l) { return l == KD_VEC_ROWS || l == KD_VEC_COLUMNS; }
 
+// Output rows that can be written in 16-byte stores (W_hat of kd_reconstruct).
+bool rows_vec_ok(const void* out, int dtype, int layout, int64_t n, int64_t ld) {
+  const int64_t esz = dtype == KD_F32 ? 4 : 2;
+  return layout == KD_VEC_ROWS && aligned_to(out, 16) && (ld * esz) % 16 == 0 && (n * esz) % 16 == 0;
+}
+
 // A matrix whose vectors are contiguous rows starting on 16-byte boundaries: the
 // decomposition stages each pair's rows into shared memory with bulk copies.
 bool rows_bulk_ok(const void* w, int dtype, int layout, int64_t n, int64_t ld) {
@@ -461,6 +467,7 @@ kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const
   p.m = m;
   p.ld = ld;
   p.out = w_hat;
+  p.vec = rows_vec_ok(w_hat, out_dtype, layout, n, ld) ? 1 : 0;
   p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.npairs = (m + 1) / 2;
@@ -527,6 +534,9 @@ kd_status kd_reconstruct_batch(const kd_recmat* mats, int count, int64_t n, kd_d
   p.twt = reinterpret_cast<const float2*>(b + L.tw);
   p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
   p.npairs = npairs;
+  p.vec = 1;
+  for (int i = 0; i < count; ++i)
+    if (mats[i].m > 0 && !rows_vec_ok(mats[i].w_hat, out_dtype, layout, n, mats[i].ld)) p.vec = 0;
   const int per = ops->ctas_per_sm(2, n);
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return KD_ERR_CUDA;

@@ -768,6 +768,9 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) apply_p_kernel(ApplyPar
 // ---------------------------------------------------------------------------
 struct RecParams {
   int dtype, layout;
+  // 1: every output row (KD_VEC_ROWS) starts 16-byte aligned and n * element size is a
+  // multiple of 16: W_hat leaves in 16-byte stores
+  int vec;
   const uint32_t* codes_u;
   const uint32_t* codes_v;
   const float* centres_u;
@@ -801,6 +804,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
   constexpr int T = PL::T;
   constexpr int E = PL::E;
   constexpr int WPV = N / 16;
+  constexpr int WPT = (WPV + T - 1) / T;  // code words per thread and plane/vector
   extern __shared__ __align__(16) float2 smem[];
   const int team = threadIdx.x / T;
   const int lt = threadIdx.x - team * T;
@@ -808,25 +812,52 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
   float2* buf = cta_setup<PL>(smem, p.twt, tw, team);
   Xform<PL, false> xf;  // scalar roots: no registers to spare for constant pairs
   xf.init(buf, tw, p.eps, lt);
-  int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
-  for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += (int64_t)gridDim.x * PL::Q) {
-    const int64_t pair = base + team;
-    const bool active = pair < p.npairs;
-    int64_t pr = active ? pair : base;
-    // this pair's matrix: index mi into rb (batched launch) or RecParams' matrix; its
-    // fields are re-read from the parameter space where used
-    int mi = 0;
-    const bool batched = PL::BATCH && rb.count > 0;
+  const bool batched = PL::BATCH && rb.count > 0;
+  // global pair -> (matrix, pair within it)
+  auto locate = [&](int64_t gp, int& mi, int64_t& pr) {
+    mi = 0;
+    pr = gp;
     if (batched) {
       while (mi + 1 < rb.count && pr >= rb.mat[mi + 1].pair0) ++mi;
       pr -= rb.mat[mi].pair0;
-      if (mi != cur_mat) {  // uniform per team: Q == 1 whenever T > 32
-        xf.set_eps(p.eps + (int64_t)mi * ((N + 31) / 32));
-        cur_mat = mi;
-      }
     }
+  };
+  // the pair's code words (uA, uB, vA, vB) of this thread, held in registers: the next
+  // pair's are loaded while the current pair is transformed
+  uint4 cw_next[WPT];
+  auto load_codes = [&](int64_t gp) {
+    int mi;
+    int64_t pr;
+    locate(gp, mi, pr);
     const uint32_t* codes_u = batched ? rb.mat[mi].codes_u : p.codes_u;
     const uint32_t* codes_v = batched ? rb.mat[mi].codes_v : p.codes_v;
+    const int64_t m_in = batched ? rb.mat[mi].m : p.m;
+    const int64_t cA = 2 * pr;
+    const int64_t cB = (cA + 1) < m_in ? cA + 1 : cA;
+#pragma unroll
+    for (int k = 0; k < WPT; ++k) {
+      const int w = lt + k * T;
+      cw_next[k] = w < WPV ? make_uint4(__ldg(&codes_u[cA * WPV + w]), __ldg(&codes_u[cB * WPV + w]),
+                                        __ldg(&codes_v[cA * WPV + w]), __ldg(&codes_v[cB * WPV + w]))
+                           : make_uint4(0u, 0u, 0u, 0u);
+    }
+  };
+  const int64_t stride = (int64_t)gridDim.x * PL::Q;
+  {
+    const int64_t base0 = (int64_t)blockIdx.x * PL::Q;
+    if (base0 < p.npairs) load_codes(base0 + team < p.npairs ? base0 + team : base0);
+  }
+  int cur_mat = 0;  // matrix whose sign set the transform holds (batch launches)
+  for (int64_t base = (int64_t)blockIdx.x * PL::Q; base < p.npairs; base += stride) {
+    const int64_t pair = base + team;
+    const bool active = pair < p.npairs;
+    int mi;
+    int64_t pr;
+    locate(active ? pair : base, mi, pr);
+    if (batched && mi != cur_mat) {  // uniform per team: Q == 1 whenever T > 32
+      xf.set_eps(p.eps + (int64_t)mi * ((N + 31) / 32));
+      cur_mat = mi;
+    }
     const float* centres_u = batched ? rb.mat[mi].centres_u : p.centres_u;
     const float* centres_v = batched ? rb.mat[mi].centres_v : p.centres_v;
     const int64_t m_in = batched ? rb.mat[mi].m : p.m;
@@ -845,9 +876,10 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
     };
     // code words of the pair staged in shared memory, word w as (uA, uB, vA, vB)
     uint4* cw = reinterpret_cast<uint4*>(buf);
-    for (int w = lt; w < WPV; w += T) {
-      cw[w] = make_uint4(__ldg(&codes_u[colA * WPV + w]), __ldg(&codes_u[colB * WPV + w]),
-                         __ldg(&codes_v[colA * WPV + w]), __ldg(&codes_v[colB * WPV + w]));
+#pragma unroll
+    for (int k = 0; k < WPT; ++k) {
+      const int w = lt + k * T;
+      if (w < WPV) cw[w] = cw_next[k];
     }
     team_sync<PL>();
     float2 uq[E], vq[E];
@@ -859,6 +891,8 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
       uq[j] = make_float2(pick(cuA, (c.x >> sh) & 3u), pick(cuB, (c.y >> sh) & 3u));
       vq[j] = make_float2(pick(cvA, (c.z >> sh) & 3u), pick(cvB, (c.w >> sh) & 3u));
     }
+    // the next pair's code words, in flight during this pair's transform
+    if (base + stride < p.npairs) load_codes(base + stride + team < p.npairs ? base + stride + team : base + stride);
     team_sync<PL>();  // the transform reuses buf
     xf.apply(vq);
     // W_hat = U_q + P V_q, staged in natural order so the stores are contiguous
@@ -872,13 +906,49 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
     if (active) {
       void* out = batched ? rb.mat[mi].out : p.out;
       const int64_t ld = batched ? rb.mat[mi].ld : p.ld;
-      for (int i = 2 * lt; i < N; i += 2 * T) {
-        const float2 e0 = buf[i], e1 = buf[i + 1];   // entries i, i + 1 of (A, B)
-        store_elem(out, p.dtype, elem_index(p.layout, colA, i, ld), e0.x);
-        store_elem(out, p.dtype, elem_index(p.layout, colA, i + 1, ld), e1.x);
-        if (hasB) {
-          store_elem(out, p.dtype, elem_index(p.layout, colB, i, ld), e0.y);
-          store_elem(out, p.dtype, elem_index(p.layout, colB, i + 1, ld), e1.y);
+      if (p.vec) {
+        // 16-byte chunks of consecutive entries: 8 at 16-bit output, 4 at fp32
+        const int per = p.dtype == DT_F32 ? 4 : 8;
+        for (int i0 = per * lt; i0 < N; i0 += per * T) {
+          float a[8], b[8];
+#pragma unroll
+          for (int e = 0; e < 8; ++e) {
+            const float2 v = e < per ? buf[i0 + e] : make_float2(0.f, 0.f);
+            a[e] = v.x;
+            b[e] = v.y;
+          }
+          auto pack = [&](const float (&f)[8]) -> uint4 {
+            if (p.dtype == DT_F32) {
+              return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
+                                __float_as_uint(f[3]));
+            }
+            uint32_t w4[4];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+              if (p.dtype == DT_F16) {
+                const __half2 t = __floats2half2_rn(f[2 * h], f[2 * h + 1]);
+                w4[h] = *reinterpret_cast<const uint32_t*>(&t);
+              } else {
+                const __nv_bfloat162 t = __floats2bfloat162_rn(f[2 * h], f[2 * h + 1]);
+                w4[h] = *reinterpret_cast<const uint32_t*>(&t);
+              }
+            }
+            return make_uint4(w4[0], w4[1], w4[2], w4[3]);
+          };
+          const int esz = p.dtype == DT_F32 ? 4 : 2;
+          char* o = static_cast<char*>(out);
+          *reinterpret_cast<uint4*>(o + (colA * ld + i0) * esz) = pack(a);
+          if (hasB) *reinterpret_cast<uint4*>(o + (colB * ld + i0) * esz) = pack(b);
+        }
+      } else {
+        for (int i = 2 * lt; i < N; i += 2 * T) {
+          const float2 e0 = buf[i], e1 = buf[i + 1];   // entries i, i + 1 of (A, B)
+          store_elem(out, p.dtype, elem_index(p.layout, colA, i, ld), e0.x);
+          store_elem(out, p.dtype, elem_index(p.layout, colA, i + 1, ld), e1.x);
+          if (hasB) {
+            store_elem(out, p.dtype, elem_index(p.layout, colB, i, ld), e0.y);
+            store_elem(out, p.dtype, elem_index(p.layout, colB, i + 1, ld), e1.y);
+          }
         }
       }
     }
