@@ -813,6 +813,20 @@ def run_profile_case(args) -> None:
         torch.cuda.synchronize()
         log(f"[profile-case] ok: {args.profile_kernel} n={spec.N} m={spec.M}")
         return
+    if args.profile_kernel == "fold":
+        # the layer's 2-bit products at batch 1 (one kd_matmul_2bit_batch), three times
+        decs = []
+        for s_ in layer_fn(0):
+            w_ = synth.generate(s_, device="cuda")
+            decs.append((s_, kd.decompose(w_, args.iters, s_.sign_seed)))
+            del w_
+        xs = {n: torch.randn((1, n), device="cuda") for n in {s_.N for s_, _ in decs}}
+        xps = [kd.apply_p(xs[s_.N], s_.sign_seed) for s_, _ in decs]
+        for _ in range(3):
+            kd.matmul_2bit_batch([d for _, d in decs], [xs[s_.N] for s_, _ in decs], xps)
+        torch.cuda.synchronize()
+        log("[profile-case] ok: fold, 7B layer, batch 1")
+        return
     if args.profile_kernel == "rht":
         y = torch.empty(w.shape, dtype=torch.float32, device="cuda")
         for _ in range(3):
@@ -847,7 +861,7 @@ def main():
     ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
     ap.add_argument("--profile-m", type=int, default=32768)
     ap.add_argument("--profile-matrix", type=int, default=0, help="layer matrix index (0 = q, 6 = down)")
-    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht", "reconstruct", "dequantise"])
+    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht", "reconstruct", "dequantise", "fold"])
     args = ap.parse_args()
     if args.profile_case:
         run_profile_case(args)

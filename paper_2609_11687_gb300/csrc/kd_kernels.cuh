@@ -895,12 +895,15 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
     if (base + stride < p.npairs) load_codes(base + stride + team < p.npairs ? base + stride + team : base + stride);
     team_sync<PL>();  // the transform reuses buf
     xf.apply(vq);
-    // W_hat = U_q + P V_q, staged in natural order so the stores are contiguous
+    // W_hat = U_q + P V_q, staged in natural order so the stores are contiguous; one
+    // spare slot per 16 keeps the 8-entry runs the 16-byte stores read conflict-free
+    auto sp = [](int i) { return i + (i >> 4); };
+    static_assert(N + N / 16 <= PL::BUF, "natural-order staging fits the exchange buffer");
     team_sync<PL>();
 #pragma unroll
     for (int j = 0; j < E; ++j) {
       const int nat = nat_of<N>(lt + j * T);
-      buf[nat] = make_float2(__fadd_rn(uq[j].x, vq[j].x), __fadd_rn(uq[j].y, vq[j].y));
+      buf[sp(nat)] = make_float2(__fadd_rn(uq[j].x, vq[j].x), __fadd_rn(uq[j].y, vq[j].y));
     }
     team_sync<PL>();
     if (active) {
@@ -913,7 +916,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
           float a[8], b[8];
 #pragma unroll
           for (int e = 0; e < 8; ++e) {
-            const float2 v = e < per ? buf[i0 + e] : make_float2(0.f, 0.f);
+            const float2 v = e < per ? buf[sp(i0 + e)] : make_float2(0.f, 0.f);
             a[e] = v.x;
             b[e] = v.y;
           }
@@ -942,7 +945,7 @@ __global__ void __launch_bounds__(PL::THREADS, PL::MINB) reconstruct_kernel(RecP
         }
       } else {
         for (int i = 2 * lt; i < N; i += 2 * T) {
-          const float2 e0 = buf[i], e1 = buf[i + 1];   // entries i, i + 1 of (A, B)
+          const float2 e0 = buf[sp(i)], e1 = buf[sp(i + 1)];   // entries i, i + 1 of (A, B)
           store_elem(out, p.dtype, elem_index(p.layout, colA, i, ld), e0.x);
           store_elem(out, p.dtype, elem_index(p.layout, colA, i + 1, ld), e1.x);
           if (hasB) {
