@@ -269,6 +269,22 @@ struct Xform {
   // passes 1 and 2, forward and inverse, stays inside a half-warp.
   static constexpr bool L12 = NP == 3 && !PL::PAIRED && PL::R(1) == 16 && PL::S(1) == 16 && PL::RL == 16 &&
                               T % 16 == 0;
+  // Warp-local units for an odd first radix (n = 11008 = 43 x 16 x 16): after pass 0
+  // the vector falls into E blocks of 256 slots, and the M partner of every frequency
+  // of block b lies in block E - b (block 0 pairs with itself).  Unit 0 is block 0,
+  // unit u >= 1 the blocks u and E - u; warp w takes units w, w + NW, ...  In a unit,
+  // lane l < 16 takes group i = l of the first block and lane l >= 16 group 31 - l of
+  // the second, in pass 1, the last pass and their inverses; M then pairs lane l with
+  // lane l ^ 16 (register 15 - k2) in registers, as the paired plans do (unit 0: lane l
+  // with lane 16 - l, lane 0 with itself).  Only the exchanges into pass 1 and out of
+  // the inverse pass 1 cross warps: two CTA barriers per P instead of five.
+  static constexpr bool WLU = NP == 3 && !PL::PAIRED && (E % 2 == 1) && PL::R(1) == 16 && PL::RL == 16 &&
+                              PL::S(1) == 16 && T == 256;
+  static constexpr int NU = (E + 1) / 2;  // units
+  static constexpr int NWT = T >= 32 ? T / 32 : 1;  // warps of the team
+  static constexpr int UPW = (NU + NWT - 1) / NWT;  // units per warp, at most
+  float2 ucw[WLU ? UPW : 1];              // per unit: exp(i pi K / N) of the lane's group K
+  uint32_t umk[WLU ? UPW : 1];            // per unit: eps_k < 0 bits (low 16), eps_{N-k} < 0 bits (high 16)
   int g1;                      // warp-local: this thread's pass-1 group
   int p0, p1;                  // slot-order M: partner slot constants
   int pb0;                     // pad(lt): base of the pass-0 slots lt + j T
@@ -303,6 +319,16 @@ struct Xform {
       lbase = slot_low<PL>(kgrp);
       cw = expi_pi(kgrp, N);
       p0 = p1 = pbp0 = pbp1 = 0;
+    } else if constexpr (WLU) {
+#pragma unroll
+      for (int q = 0; q < UPW; ++q) {
+        int b, i;
+        bool act;
+        unit_of(q, b, i, act);
+        ucw[q] = expi_pi(b + (long long)E * i, N);
+      }
+      cw = make_float2(0.f, 0.f);
+      p0 = p1 = pbp0 = pbp1 = kgrp = self = lbase = g1 = 0;
     } else {
       const int Kp = rest_of_slot<PL>(lt);
       p0 = slot_rest<PL>((T - Kp) % T);
@@ -315,6 +341,22 @@ struct Xform {
     set_eps(eb);
   }
 
+  // warp-local units: this lane's block b and group index i in its unit q (act false
+  // for the idle half of unit 0 and for units past the last)
+  __device__ __forceinline__ void unit_of(int q, int& b, int& i, bool& act) const {
+    const int w = lt >> 5, l = lt & 31;
+    const int u = w + NWT * q;
+    if (u == 0) {
+      b = 0;
+      i = l & 15;
+      act = l < 16;
+    } else {
+      b = l < 16 ? u : E - u;
+      i = l < 16 ? l : 31 - l;
+      act = u < NU;
+    }
+  }
+
   // the sign set's bits at this thread's frequencies (and their mirrors)
   __device__ __forceinline__ void set_eps(const uint32_t* __restrict__ eb) {
     ek = em = 0;
@@ -324,6 +366,22 @@ struct Xform {
         const int k = kgrp + T * kp;
         ek |= (Mask)eps_neg(eb, k) << kp;
         em |= (Mask)eps_neg(eb, (N - k) % N) << kp;
+      }
+    } else if constexpr (WLU) {
+#pragma unroll
+      for (int q = 0; q < UPW; ++q) {
+        int b, i;
+        bool act;
+        unit_of(q, b, i, act);
+        uint32_t m = 0;
+        if (b + E * i < N) {
+          for (int kp = 0; kp < 16; ++kp) {
+            const int k = b + E * i + (N / 16) * kp;
+            m |= (uint32_t)eps_neg(eb, k) << kp;
+            m |= (uint32_t)eps_neg(eb, (N - k) % N) << (16 + kp);
+          }
+        }
+        umk[q] = m;
       }
     } else {
       const int Kp = rest_of_slot<PL>(lt);
@@ -355,6 +413,19 @@ struct Xform {
     const float2 sel = diff ? t : a;
     // +-1/N with the sign of eps_k taken straight from its bit
     const uint32_t sgn = (uint32_t)((ek >> BIT) & 1u) << 31;
+    const float f = __uint_as_float(__float_as_uint(kInvN) | sgn);
+    return __fmul2_rn(sel, make_float2(f, f));
+  }
+
+  // mfreq with explicit per-group constants (warp-local units): c = exp(i pi K / N),
+  // m = the eps bits of the group's frequencies (low 16) and of their mirrors (high 16)
+  template <int KP>
+  __device__ __forceinline__ float2 mfreq_u(float2 a, float2 b, float2 c, uint32_t m) const {
+    const float2 wk = mul_root<+1, KP, 2 * 16, PK>(c);
+    const float2 t = cmul(b, wk);
+    const bool diff = ((m ^ (m >> 16)) >> KP) & 1u;
+    const float2 sel = diff ? t : a;
+    const uint32_t sgn = ((m >> KP) & 1u) << 31;
     const float f = __uint_as_float(__float_as_uint(kInvN) | sgn);
     return __fmul2_rn(sel, make_float2(f, f));
   }
@@ -435,25 +506,109 @@ struct Xform {
     // warp-local plans: pass 1 has one group per thread, in one of the warp's blocks
     constexpr bool ONE = WL && I == 1;
     for (int g = ONE ? g1 : lt; ONE || g < G; g += T) {
-      const int blk = g / S;
-      const int np = g - blk * S;
-      const int base = blk * Bk + np;
-      const int pb = pad(base);
-      auto addr = [&](int j) { return SEP ? pb + pad(j * S) : pad(base + j * S); };
-      float2 v[R];
-#pragma unroll
-      for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
-      if constexpr (DIR < 0) {
-        Dft<R, -1, PK>::run(v);
-        if constexpr (!LAST) twiddle<I, S, R, -1>(v, np);
-      } else {
-        if constexpr (!LAST) twiddle<I, S, R, +1>(v, np);
-        Dft<R, +1, PK>::run(v);
-      }
-#pragma unroll
-      for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
+      pass_group<I, DIR>(g);
       if constexpr (ONE) break;
     }
+  }
+
+  // one group g of pass I: blk = g / S, np = g % S, slots blk B(I) + np + j S
+  template <int I, int DIR>
+  __device__ __forceinline__ void pass_group(int g) {
+    constexpr int R = PL::R(I);
+    constexpr int Bk = PL::B(I);
+    constexpr int S = Bk / R;
+    constexpr bool LAST = (I == NP - 1);
+    constexpr bool SEP = PL::sep_pass(I);
+    const int blk = g / S;
+    const int np = g - blk * S;
+    const int base = blk * Bk + np;
+    const int pb = pad(base);
+    auto addr = [&](int j) { return SEP ? pb + pad(j * S) : pad(base + j * S); };
+    float2 v[R];
+#pragma unroll
+    for (int j = 0; j < R; ++j) v[j] = buf[addr(j)];
+    if constexpr (DIR < 0) {
+      Dft<R, -1, PK>::run(v);
+      if constexpr (!LAST) twiddle<I, S, R, -1>(v, np);
+    } else {
+      if constexpr (!LAST) twiddle<I, S, R, +1>(v, np);
+      Dft<R, +1, PK>::run(v);
+    }
+#pragma unroll
+    for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
+  }
+
+  // warp-local unit q: pass 1, the last pass with M in registers, their inverses
+  __device__ __forceinline__ void unit(int q) {
+    constexpr int R = 16;
+    int b, i;
+    bool act;
+    unit_of(q, b, i, act);
+    const bool selfu = (lt >> 5) == 0 && q == 0;  // unit 0: block 0 pairs with itself
+    // this unit's constants (selects, not an indexed array: stays in registers)
+    float2 c = ucw[0];
+    uint32_t m = umk[0];
+#pragma unroll
+    for (int qq = 1; qq < UPW; ++qq)
+      if (q == qq) {
+        c = ucw[qq];
+        m = umk[qq];
+      }
+    if (act) pass_group<1, -1>(16 * b + i);
+    __syncwarp();
+    // last pass: the group (b, k1 = i) at slots 256 b + 16 i + k2, frequencies
+    // b + E i + (N / 16) k2
+    constexpr bool SEP = PL::sep_pass(2);
+    const int base = PL::B(1) * b + R * i;
+    const int pb = pad(base);
+    auto addr = [&](int j) { return SEP ? pb + pad(j) : pad(base + j); };
+    float2 v[R];
+#pragma unroll
+    for (int j = 0; j < R; ++j) v[j] = act ? buf[addr(j)] : make_float2(0.f, 0.f);
+    Dft<R, -1, PK>::run(v);
+    auto body = [&](auto selfc) {
+      constexpr bool SELF = decltype(selfc)::value;
+      const int src = SELF ? (((lt & 31) < 16) ? ((16 - (lt & 31)) & 15) : (lt & 31)) : ((lt & 31) ^ 16);
+      const bool own = SELF && (lt & 31) == 0;  // frequency group 0: partners in its own registers
+      if constexpr (SELF) {
+        if (own) {
+#pragma unroll
+          for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
+        }
+      }
+      static_for<0, R / 2>([&](auto kk) {
+        constexpr int K1 = decltype(kk)::value;
+        constexpr int K2 = R - 1 - K1;
+        const float2 s1 = v[K2], s2 = v[K1];
+        float2 q1, q2;
+        q1.x = __shfl_sync(0xffffffffu, s1.x, src);
+        q1.y = __shfl_sync(0xffffffffu, s1.y, src);
+        q2.x = __shfl_sync(0xffffffffu, s2.x, src);
+        q2.y = __shfl_sync(0xffffffffu, s2.y, src);
+        if constexpr (SELF) {
+          if (own) {
+            q1 = buf[addr((R - K1) % R)];
+            q2 = buf[addr((R - K2) % R)];
+          }
+        }
+        const float2 o1 = mfreq_u<K1>(s2, q1, c, m);
+        const float2 o2 = mfreq_u<K2>(s1, q2, c, m);
+        v[K1] = o1;
+        v[K2] = o2;
+      });
+    };
+    if (selfu) {
+      body(std::true_type{});
+    } else {
+      body(std::false_type{});
+    }
+    Dft<R, +1, PK>::run(v);
+    if (act) {
+#pragma unroll
+      for (int j = 0; j < R; ++j) buf[addr(j)] = v[j];
+    }
+    __syncwarp();
+    if (act) pass_group<1, +1>(16 * b + i);
   }
 
   // paired last pass: forward DFT of own group, M with the partner lane, inverse DFT.
@@ -551,6 +706,12 @@ struct Xform {
         pass<NP - 1 - decltype(ii)::value, +1>();
         team_sync<PL>();
       });
+    } else if constexpr (WLU) {
+#pragma unroll 1
+      for (int q = 0; q < UPW; ++q) {
+        if ((lt >> 5) + NWT * q < NU) unit(q);  // warp-uniform
+      }
+      team_sync<PL>();
     } else {
       static_for<1, NP>([&](auto ii) {
         constexpr int I = decltype(ii)::value;

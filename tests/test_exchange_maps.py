@@ -118,3 +118,68 @@ def test_rht_exchange_locality(log_b, inverse):
         if kp == 1 and ki >= 2:   # write-after-read inside the half-warp
             assert all(prev_reader[slot] // 16 == t // 16 for slot, t in writer.items() if slot in prev_reader)
         prev_reader = reader
+
+
+# n = 11008 = 43 x 16 x 16 with warp-local units: after the 43-point pass the vector
+# falls into 43 blocks of 256 slots (one per pass-0 output digit b); the M partner of
+# every frequency of block b lies in block 43 - b (block 0 pairs with itself).  Unit 0
+# is block 0, unit u >= 1 the blocks u and 43 - u; warp w takes units w, w + 8, w + 16.
+# In a unit, lane l < 16 takes group i = l of the first block and lane l >= 16 group
+# i = 31 - l of the second (unit 0: lanes 0..15 only).  Pass 1 works on the group
+# (block b, np = i) at slots 256 b + i + 16 j, the last pass on the group (b, k1 = i)
+# at slots 256 b + 16 i + k2, holding frequencies b + 43 i + 688 k2.
+
+def units_11008():
+    """(warp, q, lane, block, i, active) for every unit a warp processes."""
+    out = []
+    for w in range(8):
+        for q in range(3):
+            u = w + 8 * q
+            if u >= 22:
+                continue
+            for l in range(32):
+                if u == 0:
+                    out.append((w, q, l, 0, l % 16, l < 16))
+                else:
+                    out.append((w, q, l, u if l < 16 else 43 - u, l if l < 16 else 31 - l, True))
+    return out
+
+
+def test_n11008_units_cover_every_group_once():
+    seen = [(b, i) for (_, _, _, b, i, act) in units_11008() if act]
+    assert sorted(seen) == [(b, i) for b in range(43) for i in range(16)]
+
+
+def test_n11008_partners_in_registers():
+    n = 11008
+    by = {(w, q, l): (b, i, act) for (w, q, l, b, i, act) in units_11008()}
+    for (w, q, l), (b, i, act) in by.items():
+        if not act:
+            continue
+        u = w + 8 * q
+        for k2 in range(16):
+            k = b + 43 * i + 688 * k2
+            if u == 0:
+                if i == 0:       # own register (16 - k2) % 16
+                    assert (n - k) % n == 688 * ((16 - k2) % 16)
+                else:            # lane 16 - l, register 15 - k2
+                    b2, i2, _ = by[(w, q, 16 - l)]
+                    assert b2 + 43 * i2 + 688 * (15 - k2) == n - k
+            else:                # lane l ^ 16, register 15 - k2
+                b2, i2, _ = by[(w, q, l ^ 16)]
+                assert b2 + 43 * i2 + 688 * (15 - k2) == n - k
+
+
+def test_n11008_unit_accesses_conflict_free():
+    """Every half-warp access of pass 1 (per j) and of the last pass (per k2) hits 16
+    distinct bank pairs (8-byte slots: 32 four-byte banks)."""
+    groups = {}
+    for (w, q, l, b, i, act) in units_11008():
+        if act:
+            groups.setdefault((w, q, l // 16), []).append((b, i))
+    for g in groups.values():
+        for j in range(16):
+            banks = {(2 * pad(256 * b + i + 16 * j)) % 32 for b, i in g}
+            assert len(banks) == len(g)
+            banks = {(2 * pad(256 * b + 16 * i + j)) % 32 for b, i in g}
+            assert len(banks) == len(g)
