@@ -119,3 +119,29 @@ def test_batched_calls_equal_single_calls(kd):
         y1 = kd.matmul_2bit(d, x, xp1)
         torch.cuda.synchronize()
         assert torch.equal(xp, xp1) and torch.equal(y, y1)
+
+
+def test_matmul_2bit_strided_rows(kd):
+    """Rows of x and xp with ldx > n (and misaligned by one element, so the inputs take
+    the element-wise path) and of y with ldy > m give the same result as contiguous
+    rows, bit for bit."""
+    g = torch.Generator(device="cuda").manual_seed(12)
+    m, n, b = 70, 1536, 3
+    w = (torch.randn((m, n), generator=g, device="cuda") * 0.02).half()
+    dec = kd.decompose(w, 6, 8)
+    x = torch.randn((b, n), generator=g, device="cuda")
+    xp = kd.apply_p(x, 8)
+    ref = kd.matmul_2bit(dec, x, xp)
+    for off in (0, 1):
+        xs = torch.zeros((b, n + 40), device="cuda")
+        ps = torch.zeros((b, n + 40), device="cuda")
+        xs[:, off:off + n] = x
+        ps[:, off:off + n] = xp
+        ys = torch.full((b, m + 9), float("nan"), device="cuda")
+        st = kd.kd_matmul_2bit(dec.codes_u.data_ptr(), dec.codes_v.data_ptr(), dec.centres_u.data_ptr(),
+                               dec.centres_v.data_ptr(), n, m, xs[:, off:].data_ptr(), ps[:, off:].data_ptr(), b,
+                               n + 40, ys.data_ptr(), m + 9, torch.cuda.current_stream().cuda_stream)
+        assert st == kd.KD_OK
+        torch.cuda.synchronize()
+        assert torch.equal(ys[:, :m], ref)
+        assert torch.isnan(ys[:, m:]).all()            # nothing written past m
