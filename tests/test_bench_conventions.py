@@ -45,3 +45,25 @@ def test_profile_hash_ignores_comments(bench, tmp_path):
     other = "int f() { return 2; }\nint g();\n"
     assert bench._code_only(src) == bench._code_only(same)
     assert bench._code_only(src) != bench._code_only(other)
+
+
+def test_reference_arm_line_on_cpu():
+    """The reference arm (the CPU oracle) runs without a GPU: one JSON line with
+    impl = reference, the arm's own step time (each step one pass over the fixed
+    sample), and cpu_baseline / e2e describing the same run."""
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference", "--workload", "w256",
+                          "--steps", "2", "--warmup", "3"], capture_output=True, text=True, timeout=600, cwd=root)
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [l for l in out.stdout.splitlines() if l.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    assert d["impl"] == "reference" and d["steps"] == 2 and d["warmup"] == 3
+    assert d["value"] > 0 and d["ms_per_step"] > 0 and d["higher_is_better"] is True
+    assert d["config"]["sample_params_per_step"] == 256 * 256       # the whole 256 x 256 matrix
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["value"] == d["value"]
