@@ -460,7 +460,7 @@ struct Xform {
   __device__ __forceinline__ void fwd0(float2 (&v)[E]) {
     if constexpr (kd_is_big_prime<E>()) {
       static_assert(!PL::TW2, "row-major pass-0 table");
-      dft_prime_stream<E, -1>([&](auto jc) { return v[decltype(jc)::value]; },
+      dft_prime_pass<E, -1>([&](auto jc) { return v[decltype(jc)::value]; },
                               [&](auto kc, float2 x) {
                                 constexpr int K = decltype(kc)::value;
                                 if constexpr (K > 0) x = cmul(x, ld_tw<PL::TW_SMEM>(tw + K * T + lt));  // row-major: E odd
@@ -477,7 +477,7 @@ struct Xform {
   __device__ __forceinline__ void inv0(float2 (&v)[E]) {
     if constexpr (kd_is_big_prime<E>()) {
       // outputs go back to the thread's own slots (already read), then to registers
-      dft_prime_stream<E, +1>(
+      dft_prime_pass<E, +1>(
           [&](auto jc) {
             constexpr int J = decltype(jc)::value;
             float2 x = buf[a0<J>()];
