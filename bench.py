@@ -508,18 +508,25 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
         groups.setdefault(s.N, []).extend([(d.codes_u, d.centres_u), (d.codes_v, d.centres_v)])
     planes_out = {n: [torch.empty((c.shape[0], n), dtype=torch.float16, device=c.device) for c, _ in pl]
                   for n, pl in groups.items()}
-    def timed(fn, reps=4):
+    # a layer's code planes (about 0.1 GB) fit in L2: every repetition starts from a
+    # flushed L2 (a 256 MB write outside the timed events); the median is reported
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=layer[0][1].device)
+
+    def timed(fn, reps=6):
         evs = []
         for rep in range(reps):
             a = torch.cuda.Event(enable_timing=True)
             b = torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                flush.fill_(rep & 255)
             a.record(stream)
             fn()
             b.record(stream)
             if rep > 0:
                 evs.append((a, b))
         torch.cuda.synchronize()
-        return sum(a.elapsed_time(b) for a, b in evs) / len(evs)
+        ts = sorted(a.elapsed_time(b) for a, b in evs)
+        return ts[len(ts) // 2]
 
     # every matrix to its own output, the matrices of one vector length in one launch
     rec_groups = {}
@@ -570,14 +577,30 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
                     for _, _, wh in grp:
                         torch.matmul(x16[n], wh.T)
 
+        # the tensor-core product for fp16 activations (X and XP rounded to fp16 by torch casts
+        # outside the timed region, as the dense fp16 baseline's X is)
+        xp_all()
+        xp16 = [xp.half() for xp in xps]
+
+        def prod16_all():
+            kd.matmul_2bit_f16_batch([d for _, d in decs], [x16[s_.N] for s_, _ in decs], xp16, outs=ys,
+                                     stream=stream)
+
         ms_xp, ms_prod, ms_dense = timed(xp_all, 6), timed(prod_all, 6), timed(dense_all, 6)
-        prod_bytes = sum(2 * s.M * ((s.N + 15) // 16) * 4 + 2 * s.M * 16 + 2 * bsz * s.N * 4 + bsz * s.M * 4
-                         for s, _ in layer)
+        ms_prod16 = timed(prod16_all, 6)
+        code_bytes = sum(2 * s.M * ((s.N + 15) // 16) * 4 + 2 * s.M * 16 + bsz * s.M * 4 for s, _ in layer)
+        prod_bytes = code_bytes + sum(2 * bsz * s.N * 4 for s, _ in layer)
+        prod16_bytes = code_bytes + sum(2 * bsz * s.N * 2 for s, _ in layer)
+        hbm_pk = hbm_peak_gbs()[0]
         folded[f"batch{bsz}"] = {
             "ms_product": round(ms_prod, 4), "ms_xp": round(ms_xp, 4), "ms_total": round(ms_prod + ms_xp, 4),
             "ms_dense_fp16": round(ms_dense, 4), "bound": "hbm",
-            "achieved": round(prod_bytes / (ms_prod / 1e3) / 1e9, 1), "peak": hbm_peak_gbs()[0], "unit": "GB/s",
-            "frac": round(prod_bytes / (ms_prod / 1e3) / 1e9 / hbm_peak_gbs()[0], 4)}
+            "achieved": round(prod_bytes / (ms_prod / 1e3) / 1e9, 1), "peak": hbm_pk, "unit": "GB/s",
+            "frac": round(prod_bytes / (ms_prod / 1e3) / 1e9 / hbm_pk, 4),
+            "f16_tc": {"ms_product": round(ms_prod16, 4), "ms_total": round(ms_prod16 + ms_xp, 4),
+                       "vs_dense_fp16": round(ms_dense / ms_prod16, 2),
+                       "achieved": round(prod16_bytes / (ms_prod16 / 1e3) / 1e9, 1), "peak": hbm_pk, "unit": "GB/s",
+                       "frac": round(prod16_bytes / (ms_prod16 / 1e3) / 1e9 / hbm_pk, 4)}}
     params = sum(s.params for s, _ in layer)
     # one P (a DCT and an inverse DCT) per vector: 2 * 2 n log2 n flops, plus n adds
     import math
@@ -602,7 +625,9 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
         "matmul_2bit": {"kernel": "fold_kernel (Y = X U_q^T + XP V_q^T from the 2-bit planes: one "
                                   "kd_matmul_2bit_batch per layer and group of up to 2 rows; XP by one "
                                   "kd_apply_p_batch per vector length) against torch.matmul fp16 on W_hat "
-                                  "(cuBLAS, one call per matrix), whole layer",
+                                  "(cuBLAS, one call per matrix), whole layer; f16_tc: fold16_kernel "
+                                  "(kd_matmul_2bit_f16_batch, fp16 X and XP, mma.sync m16n8k16 with fp32 sums, "
+                                  "one launch per 16 rows); L2 flushed before every repetition, median",
                         "algorithmic_bytes": "codes 0.5 B per weight + centres + x, XP, y", "peak_basis": basis,
                         **folded},
     }
@@ -827,6 +852,21 @@ def run_profile_case(args) -> None:
         torch.cuda.synchronize()
         log("[profile-case] ok: fold, 7B layer, batch 1")
         return
+    if args.profile_kernel == "fold16":
+        # the layer's fp16 tensor-core products at batch 4 (one kd_matmul_2bit_f16_batch), three times
+        decs = []
+        for s_ in layer_fn(0):
+            w_ = synth.generate(s_, device="cuda")
+            decs.append((s_, kd.decompose(w_, args.iters, s_.sign_seed)))
+            del w_
+        xs = {n: torch.randn((4, n), device="cuda") for n in {s_.N for s_, _ in decs}}
+        xps = [kd.apply_p(xs[s_.N], s_.sign_seed).half() for s_, _ in decs]
+        x16 = {n: x.half() for n, x in xs.items()}
+        for _ in range(3):
+            kd.matmul_2bit_f16_batch([d for _, d in decs], [x16[s_.N] for s_, _ in decs], xps)
+        torch.cuda.synchronize()
+        log("[profile-case] ok: fold16, 7B layer, batch 4")
+        return
     if args.profile_kernel == "rht":
         y = torch.empty(w.shape, dtype=torch.float32, device="cuda")
         for _ in range(3):
@@ -861,7 +901,7 @@ def main():
     ap.add_argument("--profile-case", action="store_true", help="small single-matrix case for ncu")
     ap.add_argument("--profile-m", type=int, default=32768)
     ap.add_argument("--profile-matrix", type=int, default=0, help="layer matrix index (0 = q, 6 = down)")
-    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht", "reconstruct", "dequantise", "fold"])
+    ap.add_argument("--profile-kernel", default="decompose", choices=["decompose", "rht", "reconstruct", "dequantise", "fold", "fold16"])
     args = ap.parse_args()
     if args.profile_case:
         run_profile_case(args)

@@ -385,6 +385,46 @@ typedef struct kd_fold_mat {
 
 kd_status kd_matmul_2bit_batch(const kd_fold_mat* mats, int count, int64_t batch, void* stream);
 
+/* The layer product of kd_matmul_2bit for fp16 activations, on the tensor cores:
+ *   y[r*ldy + j] = sum_i h(centres_u[j][code_u(j,i)]) x[r*ldx + i]
+ *                + sum_i h(centres_v[j][code_v(j,i)]) xp[r*ldx + i],   r < batch, j < m,
+ * where x and xp are fp16 (IEEE binary16) and h() rounds a centre to fp16 (nearest,
+ * ties to even); products are exact and the sums are fp32 (mma.sync m16n8k16).  This
+ * is Y = X W_hat^T in the precision of a dense fp16 layer: the activations and the
+ * weights' values are fp16, nothing else is rounded.
+ *   codes_u, codes_v, centres_u, centres_v, n, m, batch, y, ldy as in kd_matmul_2bit.
+ *   x, xp   device fp16, batch rows of n inputs, row r at x + r*ldx (ldx >= n);
+ *           xp holds the rows of X P (kd_apply_p, rounded to fp16 by the caller).
+ *           2-byte aligned; 16-byte aligned rows (base and ldx a multiple of 8) take
+ *           128-bit loads.
+ * The centres must be finite in fp16 (|c| <= 65504): a code padding past n multiplies
+ * a zero input by a centre.  Every code word is read once per group of up to 16 batch
+ * rows; the sums run in a fixed order (deterministic).  Errors and empty calls as
+ * kd_matmul_2bit. */
+kd_status kd_matmul_2bit_f16(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
+                             const float* centres_v, int64_t n, int64_t m, const void* x, const void* xp,
+                             int64_t batch, int64_t ldx, float* y, int64_t ldy, void* stream);
+
+/* kd_matmul_2bit_f16 for several matrices in one launch per 16 batch rows; each
+ * descriptor as kd_matmul_2bit_f16's arguments.  mats is a HOST array of 1 <= count <=
+ * KD_MAX_BATCH descriptors.  Results equal kd_matmul_2bit_f16's per matrix, bit for bit.
+ * Errors as kd_matmul_2bit_batch. */
+typedef struct kd_fold_mat_f16 {
+  const uint32_t* codes_u;
+  const uint32_t* codes_v;
+  const float* centres_u;
+  const float* centres_v;
+  const void* x;
+  const void* xp;
+  float* y;
+  int64_t n;
+  int64_t m;
+  int64_t ldx;
+  int64_t ldy;
+} kd_fold_mat_f16;
+
+kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int count, int64_t batch, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:
  * the weights are rotated by a randomized Hadamard transform before the

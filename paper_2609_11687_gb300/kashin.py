@@ -32,7 +32,8 @@ KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_workspace_size", "kd_signs",
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_read_status_static", "kd_staging_size_host", "kd_decompose_batch_host",
-           "kd_matmul_2bit", "kd_matmul_2bit_batch", "kd_apply_p_batch",
+           "kd_matmul_2bit", "kd_matmul_2bit_batch", "kd_matmul_2bit_f16", "kd_matmul_2bit_f16_batch",
+           "kd_apply_p_batch",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
@@ -62,6 +63,11 @@ class KdFoldMat(ctypes.Structure):
                 ("centres_v", ctypes.c_void_p), ("x", ctypes.c_void_p), ("xp", ctypes.c_void_p),
                 ("y", ctypes.c_void_p), ("n", ctypes.c_int64), ("m", ctypes.c_int64), ("ldx", ctypes.c_int64),
                 ("ldy", ctypes.c_int64)]
+
+
+class KdFoldMatF16(ctypes.Structure):
+    """Mirror of kd_fold_mat_f16 (include/kashin.h): one matrix of kd_matmul_2bit_f16_batch."""
+    _fields_ = KdFoldMat._fields_
 
 
 class KdMatrixHost(ctypes.Structure):
@@ -120,6 +126,11 @@ def _load() -> ctypes.CDLL:
     lib.kd_matmul_2bit.restype = c_int
     lib.kd_matmul_2bit_batch.argtypes = [c_vp, c_int, c_i64, c_vp]
     lib.kd_matmul_2bit_batch.restype = c_int
+    lib.kd_matmul_2bit_f16.argtypes = [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_vp, c_vp, c_i64, c_i64, c_vp, c_i64,
+                                       c_vp]
+    lib.kd_matmul_2bit_f16.restype = c_int
+    lib.kd_matmul_2bit_f16_batch.argtypes = [c_vp, c_int, c_i64, c_vp]
+    lib.kd_matmul_2bit_f16_batch.restype = c_int
     lib.kd_apply_p_batch.argtypes = [c_vp, c_int, c_i64, c_vp, c_sz, c_vp]
     lib.kd_apply_p_batch.restype = c_int
     lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
@@ -441,6 +452,48 @@ def matmul_2bit(dec: "Decomposed", x, xp, out=None, stream=None):
 
 def kd_matmul_2bit_batch(mats, count, batch, stream) -> int:
     return lib.kd_matmul_2bit_batch(mats, count, batch, stream)
+
+
+def kd_matmul_2bit_f16(codes_u, codes_v, centres_u, centres_v, n, m, x, xp, batch, ldx, y, ldy, stream) -> int:
+    return lib.kd_matmul_2bit_f16(codes_u, codes_v, centres_u, centres_v, n, m, x, xp, batch, ldx, y, ldy, stream)
+
+
+def kd_matmul_2bit_f16_batch(mats, count, batch, stream) -> int:
+    return lib.kd_matmul_2bit_f16_batch(mats, count, batch, stream)
+
+
+def matmul_2bit_f16(dec: "Decomposed", x, xp, out=None, stream=None):
+    """kd_matmul_2bit_f16: ``Y = X W_hat^T`` from the code planes on the tensor cores,
+    for fp16 ``x`` and ``xp`` (batch, n) CUDA tensors; returns (batch, m) fp32."""
+    return matmul_2bit_f16_batch([dec], [x], [xp], outs=None if out is None else [out], stream=stream)[0]
+
+
+def matmul_2bit_f16_batch(decs, xs, xps, outs=None, stream=None):
+    """kd_matmul_2bit_f16_batch: ``Y_i = X_i W_hat_i^T`` for several matrices, fp16
+    inputs (one batch size), one launch per 16 batch rows."""
+    torch = _torch()
+    if not 1 <= len(decs) <= KD_MAX_BATCH or len(xs) != len(decs) or len(xps) != len(decs):
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices with one x and one xp each")
+    b = xs[0].shape[0]
+    arr = (KdFoldMatF16 * len(decs))()
+    res = []
+    for i, (d, x, xp) in enumerate(zip(decs, xs, xps)):
+        m, words = d.codes_u.shape
+        if x.dim() != 2 or x.shape[0] != b or x.dtype != torch.float16 or xp.shape != x.shape \
+                or xp.dtype != x.dtype or x.stride(1) != 1 or xp.stride(1) != 1 or x.stride(0) != xp.stride(0):
+            raise ValueError("x and xp must be fp16 (batch, n) tensors of one shape, unit inner stride")
+        n = x.shape[1]
+        if (n + 15) // 16 != words:
+            raise ValueError("x does not match the code planes' vector length")
+        y = outs[i] if outs is not None else torch.empty((b, m), dtype=torch.float32, device=x.device)
+        arr[i] = KdFoldMatF16(d.codes_u.data_ptr(), d.codes_v.data_ptr(), d.centres_u.data_ptr(),
+                              d.centres_v.data_ptr(), x.data_ptr(), xp.data_ptr(), y.data_ptr(), n, m, x.stride(0),
+                              y.stride(0))
+        res.append(y)
+    st = kd_matmul_2bit_f16_batch(ctypes.cast(arr, ctypes.c_void_p), len(decs), b, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_matmul_2bit_f16_batch")
+    return res
 
 
 def kd_apply_p_batch(mats, count, n, workspace, ws_bytes, stream) -> int:

@@ -316,6 +316,33 @@ def test_matmul_2bit_validation(kd):
     assert f(null, null, null, null, 256, 4, null, null, 0, 256, null, 4, null) == kd.KD_OK    # batch == 0
 
 
+def test_matmul_2bit_f16_validation(kd):
+    """kd_matmul_2bit_f16 refuses bad sizes, null and unaligned pointers (fp16 rows need
+    2-byte alignment) without a CUDA call; its batched form refuses bad counts."""
+    f = kd.kd_matmul_2bit_f16
+    null = None
+    assert f(16, 16, 16, 16, 0, 4, 16, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG       # n = 0
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, 1, 255, 16, 4, null) == kd.KD_ERR_INVALID_ARG     # ldx < n
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, 1, 256, 16, 3, null) == kd.KD_ERR_INVALID_ARG     # ldy < m
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, -1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG    # batch < 0
+    assert f(16, 16, 16, 16, 256, 4, 16, null, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG   # xp null
+    assert f(16, 16, 16, 8, 256, 4, 16, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG      # centres 8-aligned
+    assert f(16, 16, 16, 16, 256, 4, 17, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG     # x odd address
+    assert f(16, 16, 16, 16, 256, 4, 16, 16, 1, 256, 18, 4, null) == kd.KD_ERR_INVALID_ARG     # y unaligned
+    assert f(null, null, null, null, 256, 0, null, null, 1, 256, null, 0, null) == kd.KD_OK    # m == 0
+    assert f(null, null, null, null, 256, 4, null, null, 0, 256, null, 4, null) == kd.KD_OK    # batch == 0
+    mats = (kd.KdFoldMatF16 * 2)()
+    mats[0] = kd.KdFoldMatF16(16, 16, 16, 16, 16, 16, 16, 256, 4, 256, 4)
+    mats[1] = kd.KdFoldMatF16(16, 16, 16, 16, 18, 16, 16, 256, 4, 255, 4)    # ldx < n
+    arr = ctypes.cast(mats, ctypes.c_void_p)
+    assert kd.kd_matmul_2bit_f16_batch(null, 1, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_f16_batch(arr, 0, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_f16_batch(arr, 33, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_f16_batch(arr, 2, 1, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_matmul_2bit_f16_batch(arr, 2, 0, null) == kd.KD_ERR_INVALID_ARG       # checked even when empty
+    assert kd.kd_matmul_2bit_f16_batch(arr, 1, 0, null) == kd.KD_OK
+
+
 def test_batched_product_and_transform_validation(kd):
     null = None
     mats = (kd.KdFoldMat * 2)()
