@@ -548,7 +548,7 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
     ms_deq = timed(deq)
 
     # the layer product straight from the 2-bit planes (one kd_matmul_2bit_batch for
-    # the layer, XP from one kd_apply_p_batch per vector length) against the dense fp16
+    # the layer, XP from one kd_apply_p_prepared per vector length) against the dense fp16
     # product on the reconstructed W_hat (cuBLAS through torch.matmul), per batch of
     # activation rows
     dev = layer[0][1].device
@@ -563,10 +563,17 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
         ys = [torch.empty((bsz, s_.M), device=dev, dtype=torch.float32) for s_, _ in decs]
         x16 = {n: x.half() for n, x in xs.items()}
 
-        def xp_all():
+        def xp_tables_all():
             for n, ix in by_n.items():
                 kd.apply_p_batch([xs[n]] * len(ix), [decs[k][0].sign_seed for k in ix], outs=[xps[k] for k in ix],
                                  workspace=wsp[n], stream=stream)
+
+        # serving: P's tables derived once per layer (kd_prepare_p), then XP per batch
+        prep = {n: kd.prepare_p(n, [decs[k][0].sign_seed for k in ix], stream=stream) for n, ix in by_n.items()}
+
+        def xp_all():
+            for n, ix in by_n.items():
+                kd.apply_p_prepared([xs[n]] * len(ix), prep[n], outs=[xps[k] for k in ix], stream=stream)
 
         def prod_all():
             kd.matmul_2bit_batch([d for _, d in decs], [xs[s_.N] for s_, _ in decs], xps, outs=ys, stream=stream)
@@ -587,13 +594,14 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
                                      stream=stream)
 
         ms_xp, ms_prod, ms_dense = timed(xp_all, 6), timed(prod_all, 6), timed(dense_all, 6)
-        ms_prod16 = timed(prod16_all, 6)
+        ms_prod16, ms_xp_tables = timed(prod16_all, 6), timed(xp_tables_all, 6)
         code_bytes = sum(2 * s.M * ((s.N + 15) // 16) * 4 + 2 * s.M * 16 + bsz * s.M * 4 for s, _ in layer)
         prod_bytes = code_bytes + sum(2 * bsz * s.N * 4 for s, _ in layer)
         prod16_bytes = code_bytes + sum(2 * bsz * s.N * 2 for s, _ in layer)
         hbm_pk = hbm_peak_gbs()[0]
         folded[f"batch{bsz}"] = {
-            "ms_product": round(ms_prod, 4), "ms_xp": round(ms_xp, 4), "ms_total": round(ms_prod + ms_xp, 4),
+            "ms_product": round(ms_prod, 4), "ms_xp": round(ms_xp, 4), "ms_xp_deriving_tables": round(ms_xp_tables, 4),
+            "ms_total": round(ms_prod + ms_xp, 4),
             "ms_dense_fp16": round(ms_dense, 4), "bound": "hbm",
             "achieved": round(prod_bytes / (ms_prod / 1e3) / 1e9, 1), "peak": hbm_pk, "unit": "GB/s",
             "frac": round(prod_bytes / (ms_prod / 1e3) / 1e9 / hbm_pk, 4),
@@ -624,7 +632,9 @@ def measure_inference(kd, torch, layer, iters, wss, stream):
                        "algorithmic_bytes_per_param": 4.5},
         "matmul_2bit": {"kernel": "fold_kernel (Y = X U_q^T + XP V_q^T from the 2-bit planes: one "
                                   "kd_matmul_2bit_batch per layer and group of up to 2 rows; XP by one "
-                                  "kd_apply_p_batch per vector length) against torch.matmul fp16 on W_hat "
+                                  "kd_apply_p_prepared per vector length on tables kd_prepare_p derived once "
+                                  "per layer; ms_xp_deriving_tables: kd_apply_p_batch, tables derived per call) "
+                                  "against torch.matmul fp16 on W_hat "
                                   "(cuBLAS, one call per matrix), whole layer; f16_tc: fold16_kernel "
                                   "(kd_matmul_2bit_f16_batch, fp16 X and XP, mma.sync m16n8k16 with fp32 sums, "
                                   "one launch per 16 rows); L2 flushed before every repetition, median",

@@ -266,6 +266,20 @@ typedef struct kd_pmat {
 kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
                            void* stream);
 
+/* P's tables derived once, for serving: kd_prepare_p writes the twiddle table and the
+ * sign sets of seeds[0..count) (set i from seeds[i]) into the workspace, on `stream`;
+ * kd_apply_p_prepared then applies P to the rows of each matrix as kd_apply_p_batch does,
+ * matrix i with sign set i, without deriving the tables again (its descriptors'
+ * sign_seed fields are not read).  The two calls take the same n, count and workspace
+ * (16-byte aligned, ws_bytes >= kd_workspace_size_batch(n, count)); results equal
+ * kd_apply_p_batch's with the same seeds, bit for bit.  The tables stay valid until
+ * another call writes that workspace.  Errors as kd_apply_p_batch (seeds null:
+ * KD_ERR_INVALID_ARG). */
+kd_status kd_prepare_p(const uint64_t* seeds, int count, int64_t n, void* workspace, size_t ws_bytes,
+                       void* stream);
+kd_status kd_apply_p_prepared(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
+                              void* stream);
+
 /* Dense re-materialisation W_hat = U_q + P V_q (App. C): vector j of w_hat is
  * centres_u[j][code_u] + P(centres_v[j][code_v]).  Inputs as produced by
  * kd_decompose (centres 16-byte aligned, codes 4-byte aligned, KD_ERR_INVALID_ARG

@@ -383,8 +383,16 @@ kd_status kd_apply_p(const float* x, float* y, int64_t n, int64_t m, uint64_t si
   return ops->apply(p, nullptr, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
 }
 
-kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
-                           void* stream) {
+}  // extern "C"
+
+namespace kd {
+namespace {
+
+// kd_apply_p_batch and kd_apply_p_prepared: with `prepared` the workspace already holds
+// the twiddle table and sign set i of matrix i (kd_prepare_p); otherwise they are derived
+// here from the matrices' seeds first.
+kd_status apply_p_many(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes, void* stream,
+                       bool prepared) {
   if (!mats || count < 1 || count > KD_MAX_BATCH || n <= 0) return KD_ERR_INVALID_ARG;
   const PlanOps* ops = plan_ops(n);
   if (!ops) return KD_ERR_UNSUPPORTED_N;
@@ -406,7 +414,7 @@ kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* work
   if (!layout_of(ops, &L, count)) return KD_ERR_CUDA;
   if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (!ops->batch) {
+  if (!ops->batch && !prepared) {
     // long vectors and the run-time-length path: one launch per matrix, in stream order
     for (int i = 0; i < count; ++i) {
       const kd_status sti = kd_apply_p(mats[i].x, mats[i].y, n, mats[i].m, mats[i].sign_seed, workspace, ws_bytes,
@@ -415,25 +423,67 @@ kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* work
     }
     return KD_OK;
   }
-  uint64_t seeds[KD_MAX_BATCH];
-  for (int i = 0; i < count; ++i) seeds[i] = mats[i].sign_seed;
-  kd_status st = setup_batch(ops, L, workspace, seeds, count, n, s);
-  if (st != KD_OK || npairs == 0) return st;
+  if (!prepared) {
+    uint64_t seeds[KD_MAX_BATCH];
+    for (int i = 0; i < count; ++i) seeds[i] = mats[i].sign_seed;
+    const kd_status st = setup_batch(ops, L, workspace, seeds, count, n, s);
+    if (st != KD_OK) return st;
+  }
+  if (npairs == 0) return KD_OK;
   char* b = static_cast<char*>(workspace);
-  ApplyParams p;
-  std::memset(&p, 0, sizeof(p));
-  p.n = n;
-  p.m = mats[0].m;
-  p.x = mats[0].x;
-  p.y = mats[0].y;
-  p.twt = reinterpret_cast<const float2*>(b + L.tw);
-  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
-  p.npairs = npairs;
   const int per = ops->ctas_per_sm(1, n);
   const int sms = sm_count();
   if (per <= 0 || sms <= 0) return KD_ERR_CUDA;
-  const int grid = grid_for(p.npairs, ops->q, per * sms);
-  return ops->apply(p, &ab, grid, s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+  ApplyParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.n = n;
+  p.twt = reinterpret_cast<const float2*>(b + L.tw);
+  if (!ops->batch) {
+    // one launch per matrix, each on its own prepared sign set
+    const size_t words = (size_t)((n + 31) / 32);
+    for (int i = 0; i < count; ++i) {
+      if (mats[i].m == 0) continue;
+      p.m = mats[i].m;
+      p.x = mats[i].x;
+      p.y = mats[i].y;
+      p.eps = reinterpret_cast<const uint32_t*>(b + L.eps) + (size_t)i * words;
+      p.npairs = (mats[i].m + 1) / 2;
+      if (ops->apply(p, nullptr, grid_for(p.npairs, ops->q, per * sms), s) != cudaSuccess) return KD_ERR_CUDA;
+    }
+    return KD_OK;
+  }
+  p.m = mats[0].m;
+  p.x = mats[0].x;
+  p.y = mats[0].y;
+  p.eps = reinterpret_cast<const uint32_t*>(b + L.eps);
+  p.npairs = npairs;
+  return ops->apply(p, &ab, grid_for(p.npairs, ops->q, per * sms), s) == cudaSuccess ? KD_OK : KD_ERR_CUDA;
+}
+
+}  // namespace
+}  // namespace kd
+
+extern "C" {
+
+kd_status kd_apply_p_batch(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
+                           void* stream) {
+  return kd::apply_p_many(mats, count, n, workspace, ws_bytes, stream, false);
+}
+
+kd_status kd_prepare_p(const uint64_t* seeds, int count, int64_t n, void* workspace, size_t ws_bytes,
+                       void* stream) {
+  if (!seeds || count < 1 || count > KD_MAX_BATCH || n <= 0) return KD_ERR_INVALID_ARG;
+  const PlanOps* ops = plan_ops(n);
+  if (!ops) return KD_ERR_UNSUPPORTED_N;
+  WsLayout L;
+  if (!layout_of(ops, &L, count)) return KD_ERR_CUDA;
+  if (!ws_ok(workspace) || ws_bytes < L.total) return KD_ERR_WORKSPACE;
+  return setup_batch(ops, L, workspace, seeds, count, n, static_cast<cudaStream_t>(stream));
+}
+
+kd_status kd_apply_p_prepared(const kd_pmat* mats, int count, int64_t n, void* workspace, size_t ws_bytes,
+                              void* stream) {
+  return kd::apply_p_many(mats, count, n, workspace, ws_bytes, stream, true);
 }
 
 kd_status kd_reconstruct(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,

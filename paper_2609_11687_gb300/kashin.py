@@ -33,7 +33,7 @@ EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_wor
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_read_status_static", "kd_staging_size_host", "kd_decompose_batch_host",
            "kd_matmul_2bit", "kd_matmul_2bit_batch", "kd_matmul_2bit_f16", "kd_matmul_2bit_f16_batch",
-           "kd_apply_p_batch",
+           "kd_apply_p_batch", "kd_prepare_p", "kd_apply_p_prepared",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
 KD_MAX_BATCH = 32
@@ -126,6 +126,10 @@ def _load() -> ctypes.CDLL:
     lib.kd_matmul_2bit.restype = c_int
     lib.kd_matmul_2bit_batch.argtypes = [c_vp, c_int, c_i64, c_vp]
     lib.kd_matmul_2bit_batch.restype = c_int
+    lib.kd_prepare_p.argtypes = [c_vp, c_int, c_i64, c_vp, ctypes.c_size_t, c_vp]
+    lib.kd_prepare_p.restype = c_int
+    lib.kd_apply_p_prepared.argtypes = [c_vp, c_int, c_i64, c_vp, ctypes.c_size_t, c_vp]
+    lib.kd_apply_p_prepared.restype = c_int
     lib.kd_matmul_2bit_f16.argtypes = [c_vp, c_vp, c_vp, c_vp, c_i64, c_i64, c_vp, c_vp, c_i64, c_i64, c_vp, c_i64,
                                        c_vp]
     lib.kd_matmul_2bit_f16.restype = c_int
@@ -546,6 +550,49 @@ def apply_p_batch(xs, sign_seeds, outs=None, workspace: Optional[Workspace] = No
     st = kd_apply_p_batch(ctypes.cast(arr, ctypes.c_void_p), len(xs), n, ws.ptr, ws.nbytes, _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_apply_p_batch")
+    return res
+
+
+def kd_prepare_p(seeds, count, n, workspace, ws_bytes, stream) -> int:
+    return lib.kd_prepare_p(seeds, count, n, workspace, ws_bytes, stream)
+
+
+def kd_apply_p_prepared(mats, count, n, workspace, ws_bytes, stream) -> int:
+    return lib.kd_apply_p_prepared(mats, count, n, workspace, ws_bytes, stream)
+
+
+def prepare_p(n: int, sign_seeds, workspace: Optional[Workspace] = None, device="cuda", stream=None) -> Workspace:
+    """kd_prepare_p: P's twiddle table and the sign sets of ``sign_seeds`` written once
+    into a workspace (returned) for apply_p_prepared."""
+    if not 1 <= len(sign_seeds) <= KD_MAX_BATCH:
+        raise ValueError(f"1..{KD_MAX_BATCH} sign seeds")
+    ws = workspace if workspace is not None else Workspace(n, device, count=len(sign_seeds))
+    seeds = (ctypes.c_uint64 * len(sign_seeds))(*[int(s) & ((1 << 64) - 1) for s in sign_seeds])
+    st = kd_prepare_p(ctypes.cast(seeds, ctypes.c_void_p), len(sign_seeds), n, ws.ptr, ws.nbytes, _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_prepare_p")
+    return ws
+
+
+def apply_p_prepared(xs, workspace: Workspace, outs=None, stream=None):
+    """kd_apply_p_prepared: ``y_i = P_i x_i`` with the tables prepare_p left in
+    ``workspace`` (matrix i takes sign set i)."""
+    torch = _torch()
+    if not 1 <= len(xs) <= KD_MAX_BATCH:
+        raise ValueError(f"1..{KD_MAX_BATCH} matrices")
+    n = xs[0].shape[1]
+    arr = (KdPMat * len(xs))()
+    res = []
+    for i, x in enumerate(xs):
+        if x.dtype != torch.float32 or not x.is_contiguous() or x.dim() != 2 or x.shape[1] != n:
+            raise ValueError("inputs must be contiguous fp32 (m, n) CUDA tensors of one n")
+        y = outs[i] if outs is not None else torch.empty_like(x)
+        arr[i] = KdPMat(x.data_ptr(), y.data_ptr(), x.shape[0], 0)
+        res.append(y)
+    st = kd_apply_p_prepared(ctypes.cast(arr, ctypes.c_void_p), len(xs), n, workspace.ptr, workspace.nbytes,
+                             _stream(stream))
+    if st != KD_OK:
+        raise KashinError(st, "kd_apply_p_prepared")
     return res
 
 

@@ -343,6 +343,27 @@ def test_matmul_2bit_f16_validation(kd):
     assert kd.kd_matmul_2bit_f16_batch(arr, 1, 0, null) == kd.KD_OK
 
 
+def test_prepared_p_validation(kd):
+    """kd_prepare_p and kd_apply_p_prepared refuse bad counts, null arrays, bad and
+    unsupported lengths before any CUDA call."""
+    null = None
+    seeds = (ctypes.c_uint64 * 2)(1, 2)
+    sp = ctypes.cast(seeds, ctypes.c_void_p)
+    assert kd.kd_prepare_p(null, 1, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_prepare_p(sp, 0, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_prepare_p(sp, 33, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_prepare_p(sp, 2, 0, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_prepare_p(sp, 2, 4094, 16, 1 << 20, null) == kd.KD_ERR_UNSUPPORTED_N
+    pm = (kd.KdPMat * 2)()
+    pm[0] = kd.KdPMat(16, 16, 4, 0)
+    pm[1] = kd.KdPMat(16, 6, 4, 0)                                         # y not 4-byte aligned
+    parr = ctypes.cast(pm, ctypes.c_void_p)
+    assert kd.kd_apply_p_prepared(null, 1, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_apply_p_prepared(parr, 0, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+    assert kd.kd_apply_p_prepared(parr, 1, 4094, 16, 1 << 20, null) == kd.KD_ERR_UNSUPPORTED_N
+    assert kd.kd_apply_p_prepared(parr, 2, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
+
+
 def test_batched_product_and_transform_validation(kd):
     null = None
     mats = (kd.KdFoldMat * 2)()

@@ -145,3 +145,21 @@ def test_matmul_2bit_strided_rows(kd):
         torch.cuda.synchronize()
         assert torch.equal(ys[:, :m], ref)
         assert torch.isnan(ys[:, m:]).all()            # nothing written past m
+
+
+@pytest.mark.parametrize("n,ms", [(768, (37, 0, 5)), (11008, (3, 6)), (1000, (2, 7))])
+def test_prepared_p_equals_batched(kd, n, ms):
+    """kd_prepare_p once, then kd_apply_p_prepared (twice, the tables reused) equals
+    kd_apply_p_batch with the same seeds bit for bit: a batched plan with an empty
+    matrix, the one-launch-per-matrix plan of n = 11008, the run-time-length path."""
+    g = torch.Generator(device="cuda").manual_seed(n)
+    xs = [torch.randn((m, n), generator=g, device="cuda") for m in ms]
+    seeds = [11 * (i + 1) for i in range(len(ms))]
+    ref = kd.apply_p_batch(xs, seeds)
+    ws = kd.prepare_p(n, seeds)
+    for _ in range(2):
+        got = kd.apply_p_prepared(xs, ws)
+        torch.cuda.synchronize()
+        for a, b in zip(ref, got):
+            assert torch.equal(a, b)
+
