@@ -439,6 +439,15 @@ typedef struct kd_fold_mat_f16 {
 
 kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int count, int64_t batch, void* stream);
 
+/* kd_matmul_2bit_f16 and its batched form for bf16 activations: x and xp are bf16, each
+ * centre is rounded to bf16 (nearest, ties to even), products are exact and sums fp32
+ * (mma.sync m16n8k16 .bf16).  Arguments, layouts, alignment and errors as the fp16
+ * calls (the descriptor struct is shared). */
+kd_status kd_matmul_2bit_bf16(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
+                              const float* centres_v, int64_t n, int64_t m, const void* x, const void* xp,
+                              int64_t batch, int64_t ldx, float* y, int64_t ldy, void* stream);
+kd_status kd_matmul_2bit_bf16_batch(const kd_fold_mat_f16* mats, int count, int64_t batch, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Randomized-Hadamard incoherence rotation (Sec. 4, the "+H" of Kashin-DCT+H:
  * the weights are rotated by a randomized Hadamard transform before the

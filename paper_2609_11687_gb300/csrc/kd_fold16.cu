@@ -1,9 +1,10 @@
-// The folded 2-bit layer product of App. C for fp16 activations, on the tensor cores:
+// The folded 2-bit layer product of App. C for 16-bit activations (fp16 or bf16), on the
+// tensor cores:
 //
 //     y[r][j] = sum_i h(cu_j[code_u(j, i)]) x[r][i] + sum_i h(cv_j[code_v(j, i)]) xp[r][i]
 //
-// with x, xp fp16 (xp = X P from kd_apply_p, rounded by the caller), h() the fp16
-// rounding of a centre, fp32 accumulation.  Neither plane is expanded in memory: each
+// with x, xp in the 16-bit type (xp = X P from kd_apply_p, rounded by the caller), h()
+// the rounding of a centre to that type, fp32 accumulation.  Neither plane is expanded in memory: each
 // code becomes its fp16 centre in registers and feeds an mma.sync B fragment directly.
 //
 // Mapping.  mma.m16n8k16 with M = the batch rows (up to 16 per launch), N = 8 output
@@ -27,6 +28,7 @@
 // bytes) and H (their high bytes).  For two codes q0, q1 one byte permute with the
 // selector nibbles (q0, q0 + 4, q1, q1 + 4) yields the fp16 pair (c[q0], c[q1]); the
 // selectors of two k-steps are formed together from one shifted code word.
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
@@ -61,12 +63,28 @@ struct Fold16Params {
   Fold16Mat mat[KD_MAX_BATCH];
 };
 
-__device__ __forceinline__ void mma_f16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
-                                        uint32_t b0, uint32_t b1) {
-  asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
-      "{%0, %1, %2, %3};\n"
-      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+// D += A B for one m16n8k16 tile; BF: the 16-bit operands are bf16 instead of fp16
+template <bool BF>
+__device__ __forceinline__ void mma_16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                       uint32_t b0, uint32_t b1) {
+  if constexpr (BF) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  } else {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};\n"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+  }
+}
+
+// a centre rounded (nearest, ties to even) to the activations' 16-bit type, as bits
+template <bool BF>
+__device__ __forceinline__ uint32_t bits16(float c) {
+  if constexpr (BF) return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(c));
+  else return (uint32_t)__half_as_ushort(__float2half_rn(c));
 }
 
 // Byte selectors for the code nibbles at bits 0..3 (low half) and 16..19 (high half) of
@@ -78,14 +96,13 @@ __device__ __forceinline__ uint32_t selectors(uint32_t t) {
   return x * 0x11u + 0x40404040u;
 }
 
-// The fp16 centres of one channel as (low bytes, high bytes), zero past m.
+// The 16-bit centres of one channel as (low bytes, high bytes), zero past m.
+template <bool BF>
 __device__ __forceinline__ uint2 centre_bytes(const float* centres, int64_t j, bool ok) {
   if (!ok) return make_uint2(0u, 0u);
   const float4 c = __ldg(reinterpret_cast<const float4*>(centres) + j);
-  const uint32_t p01 = (uint32_t)__half_as_ushort(__float2half_rn(c.x)) |
-                       ((uint32_t)__half_as_ushort(__float2half_rn(c.y)) << 16);
-  const uint32_t p23 = (uint32_t)__half_as_ushort(__float2half_rn(c.z)) |
-                       ((uint32_t)__half_as_ushort(__float2half_rn(c.w)) << 16);
+  const uint32_t p01 = bits16<BF>(c.x) | (bits16<BF>(c.y) << 16);
+  const uint32_t p23 = bits16<BF>(c.z) | (bits16<BF>(c.w) << 16);
   return make_uint2(__byte_perm(p01, p23, 0x6420u), __byte_perm(p01, p23, 0x7531u));
 }
 
@@ -112,7 +129,7 @@ __device__ __forceinline__ void load_row16(uint32_t (&r)[8], const unsigned shor
   }
 }
 
-template <bool HI>
+template <bool HI, bool BF>
 __global__ void __launch_bounds__(kF16Threads, HI ? 3 : 4) fold16_kernel(const __grid_constant__ Fold16Params p) {
   __shared__ float red[kF16Warps][kF16Rows][kRedStride];
   const int lane = threadIdx.x & 31;
@@ -134,8 +151,8 @@ __global__ void __launch_bounds__(kF16Threads, HI ? 3 : 4) fold16_kernel(const _
     for (int nt = 0; nt < 4; ++nt) {
       const int64_t j = c0 + 8 * nt + g;
       live[nt] = j < a.m;
-      cu[nt] = centre_bytes(a.centres_u, j, live[nt]);
-      cv[nt] = centre_bytes(a.centres_v, j, live[nt]);
+      cu[nt] = centre_bytes<BF>(a.centres_u, j, live[nt]);
+      cv[nt] = centre_bytes<BF>(a.centres_v, j, live[nt]);
       ru[nt] = a.codes_u + (live[nt] ? j : 0) * a.words;
       rv[nt] = a.codes_v + (live[nt] ? j : 0) * a.words;
     }
@@ -196,8 +213,8 @@ __global__ void __launch_bounds__(kF16Threads, HI ? 3 : 4) fold16_kernel(const _
           const uint32_t bu1 = __byte_perm(cu[nt].x, cu[nt].y, s1u >> sh);
           const uint32_t bv0 = __byte_perm(cv[nt].x, cv[nt].y, s0v >> sh);
           const uint32_t bv1 = __byte_perm(cv[nt].x, cv[nt].y, s1v >> sh);
-          mma_f16(acc[nt], cax[2 * j], caxh[2 * j], cax[2 * j + 1], caxh[2 * j + 1], bu0, bu1);
-          mma_f16(acc[nt], cap[2 * j], caph[2 * j], cap[2 * j + 1], caph[2 * j + 1], bv0, bv1);
+          mma_16<BF>(acc[nt], cax[2 * j], caxh[2 * j], cax[2 * j + 1], caxh[2 * j + 1], bu0, bu1);
+          mma_16<BF>(acc[nt], cap[2 * j], caph[2 * j], cap[2 * j + 1], caph[2 * j + 1], bv0, bv1);
         }
       }
     }
@@ -239,11 +256,13 @@ kd_status check_fold16(const kd_fold_mat_f16& a, int64_t batch) {
 }  // namespace
 }  // namespace kd
 
-extern "C" kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int count, int64_t batch,
-                                              void* stream) {
+namespace kd {
+namespace {
+
+kd_status fold16_run(const kd_fold_mat_f16* mats, int count, int64_t batch, void* stream, bool bf) {
   if (!mats || count < 1 || count > KD_MAX_BATCH || batch < 0) return KD_ERR_INVALID_ARG;
   for (int i = 0; i < count; ++i) {
-    const kd_status st = kd::check_fold16(mats[i], batch);
+    const kd_status st = check_fold16(mats[i], batch);
     if (st != KD_OK) return st;
   }
   int64_t work = 0;
@@ -251,10 +270,10 @@ extern "C" kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int c
   if (batch == 0 || work == 0) return KD_OK;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
   // batch rows sixteen at a time (the mma's M): each launch reads the code planes once
-  for (int64_t b0 = 0; b0 < batch; b0 += kd::kF16Rows) {
-    kd::Fold16Params p;
+  for (int64_t b0 = 0; b0 < batch; b0 += kF16Rows) {
+    Fold16Params p;
     p.count = count;
-    p.rows = (int)(batch - b0 < kd::kF16Rows ? batch - b0 : kd::kF16Rows);
+    p.rows = (int)(batch - b0 < kF16Rows ? batch - b0 : kF16Rows);
     // work items numbered longest vectors first, so that the long items of a layer are
     // not the last ones started
     int order[KD_MAX_BATCH];
@@ -268,7 +287,7 @@ extern "C" kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int c
     int64_t items = 0;
     for (int i = 0; i < count; ++i) {
       const kd_fold_mat_f16& a = mats[order[i]];
-      kd::Fold16Mat& f = p.mat[i];
+      Fold16Mat& f = p.mat[i];
       f.codes_u = a.codes_u;
       f.codes_v = a.codes_v;
       f.centres_u = a.centres_u;
@@ -282,18 +301,37 @@ extern "C" kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int c
       f.ldx = a.ldx;
       f.ldy = a.ldy;
       f.item0 = items;
-      f.vec = kd::aligned16(f.x, 16) && kd::aligned16(f.xp, 16) && a.ldx % 8 == 0;
-      items += (a.m + kd::kF16Tile - 1) / kd::kF16Tile;
+      f.vec = aligned16(f.x, 16) && aligned16(f.xp, 16) && a.ldx % 8 == 0;
+      items += (a.m + kF16Tile - 1) / kF16Tile;
     }
     p.items = items;
     if (items == 0) continue;
     // one CTA per work item (the grid-stride loop covers grids past 2^30 items)
     const int64_t grid = items < (int64_t)1 << 30 ? items : (int64_t)1 << 30;
-    if (p.rows > 8) kd::fold16_kernel<true><<<(unsigned)grid, kd::kF16Threads, 0, s>>>(p);
-    else kd::fold16_kernel<false><<<(unsigned)grid, kd::kF16Threads, 0, s>>>(p);
+    const unsigned gr = (unsigned)grid;
+    if (bf) {
+      if (p.rows > 8) fold16_kernel<true, true><<<gr, kF16Threads, 0, s>>>(p);
+      else fold16_kernel<false, true><<<gr, kF16Threads, 0, s>>>(p);
+    } else {
+      if (p.rows > 8) fold16_kernel<true, false><<<gr, kF16Threads, 0, s>>>(p);
+      else fold16_kernel<false, false><<<gr, kF16Threads, 0, s>>>(p);
+    }
     if (cudaGetLastError() != cudaSuccess) return KD_ERR_CUDA;
   }
   return KD_OK;
+}
+
+}  // namespace
+}  // namespace kd
+
+extern "C" kd_status kd_matmul_2bit_f16_batch(const kd_fold_mat_f16* mats, int count, int64_t batch,
+                                              void* stream) {
+  return kd::fold16_run(mats, count, batch, stream, false);
+}
+
+extern "C" kd_status kd_matmul_2bit_bf16_batch(const kd_fold_mat_f16* mats, int count, int64_t batch,
+                                               void* stream) {
+  return kd::fold16_run(mats, count, batch, stream, true);
 }
 
 extern "C" kd_status kd_matmul_2bit_f16(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
@@ -302,4 +340,12 @@ extern "C" kd_status kd_matmul_2bit_f16(const uint32_t* codes_u, const uint32_t*
                                         void* stream) {
   const kd_fold_mat_f16 a{codes_u, codes_v, centres_u, centres_v, x, xp, y, n, m, ldx, ldy};
   return kd_matmul_2bit_f16_batch(&a, 1, batch, stream);
+}
+
+extern "C" kd_status kd_matmul_2bit_bf16(const uint32_t* codes_u, const uint32_t* codes_v, const float* centres_u,
+                                         const float* centres_v, int64_t n, int64_t m, const void* x,
+                                         const void* xp, int64_t batch, int64_t ldx, float* y, int64_t ldy,
+                                         void* stream) {
+  const kd_fold_mat_f16 a{codes_u, codes_v, centres_u, centres_v, x, xp, y, n, m, ldx, ldy};
+  return kd_matmul_2bit_bf16_batch(&a, 1, batch, stream);
 }

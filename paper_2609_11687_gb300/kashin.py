@@ -33,6 +33,7 @@ EXPORTS = ("kd_status_string", "kd_version", "kd_supported", "kd_tuned", "kd_wor
            "kd_decompose", "kd_apply_p", "kd_reconstruct", "kd_read_status", "kd_decompose_static",
            "kd_read_status_static", "kd_staging_size_host", "kd_decompose_batch_host",
            "kd_matmul_2bit", "kd_matmul_2bit_batch", "kd_matmul_2bit_f16", "kd_matmul_2bit_f16_batch",
+           "kd_matmul_2bit_bf16", "kd_matmul_2bit_bf16_batch",
            "kd_apply_p_batch", "kd_prepare_p", "kd_apply_p_prepared",
            "kd_rht_block", "kd_rht", "kd_dequantise", "kd_dequantise_batch", "kd_measure_fp32_peak",
            "kd_workspace_size_batch", "kd_decompose_batch", "kd_reconstruct_batch")
@@ -135,6 +136,10 @@ def _load() -> ctypes.CDLL:
     lib.kd_matmul_2bit_f16.restype = c_int
     lib.kd_matmul_2bit_f16_batch.argtypes = [c_vp, c_int, c_i64, c_vp]
     lib.kd_matmul_2bit_f16_batch.restype = c_int
+    lib.kd_matmul_2bit_bf16.argtypes = lib.kd_matmul_2bit_f16.argtypes
+    lib.kd_matmul_2bit_bf16.restype = c_int
+    lib.kd_matmul_2bit_bf16_batch.argtypes = [c_vp, c_int, c_i64, c_vp]
+    lib.kd_matmul_2bit_bf16_batch.restype = c_int
     lib.kd_apply_p_batch.argtypes = [c_vp, c_int, c_i64, c_vp, c_sz, c_vp]
     lib.kd_apply_p_batch.restype = c_int
     lib.kd_workspace_size_batch.argtypes = [c_i64, c_int]
@@ -307,6 +312,12 @@ def _ptr(t) -> Optional[int]:
     return None if t is None else t.data_ptr()
 
 
+def _ld(t) -> int:
+    """Row stride of a 2-D tensor for the C ABI: a single row's stride is never used, so
+    report its length (torch and numpy may give a one-row tensor any row stride)."""
+    return t.stride(0) if t.shape[0] > 1 else t.shape[1]
+
+
 def _stream(stream) -> int:
     torch = _torch()
     s = stream if stream is not None else torch.cuda.current_stream()
@@ -364,7 +375,7 @@ def decompose(w, iters: int, sign_seed: int, layout: str = "rows", factors: bool
         m, n = w.shape
     else:
         n, m = w.shape
-    ld = w.stride(0)
+    ld = _ld(w)
     dev = w.device
     words = (n + 15) // 16
     if out is None:
@@ -417,7 +428,7 @@ def decompose_batch(ws, iters: int, sign_seeds, layout: str = "rows", coeffs: bo
                            centres_u=torch.empty((m, 4), **f32), centres_v=torch.empty((m, 4), **f32),
                            coeffs=torch.empty((m, 4), **f32) if coeffs else None,
                            u=None, vhat=None, resid=None, trace=None)
-        arr[i] = KdMatrix(w.data_ptr(), m, w.stride(0), int(sign_seeds[i]) & ((1 << 64) - 1),
+        arr[i] = KdMatrix(w.data_ptr(), m, _ld(w), int(sign_seeds[i]) & ((1 << 64) - 1),
                           _ptr(o.codes_u), _ptr(o.codes_v), _ptr(o.centres_u), _ptr(o.centres_v), _ptr(o.coeffs))
         res.append(o)
     wsp = workspace if workspace is not None else Workspace(n, ws[0].device, count=len(ws))
@@ -440,15 +451,15 @@ def matmul_2bit(dec: "Decomposed", x, xp, out=None, stream=None):
     m, words = dec.codes_u.shape
     if x.dim() != 2 or x.dtype != torch.float32 or xp.shape != x.shape or xp.dtype != x.dtype:
         raise ValueError("x and xp must be fp32 (batch, n) tensors of one shape")
-    if x.stride(1) != 1 or xp.stride(1) != 1 or x.stride(0) != xp.stride(0):
+    if x.stride(1) != 1 or xp.stride(1) != 1 or _ld(x) != _ld(xp):
         raise ValueError("x and xp need unit inner stride and equal row strides")
     b, n = x.shape
     if (n + 15) // 16 != words:
         raise ValueError("x does not match the code planes' vector length")
     y = out if out is not None else torch.empty((b, m), dtype=torch.float32, device=x.device)
     st = kd_matmul_2bit(dec.codes_u.data_ptr(), dec.codes_v.data_ptr(), dec.centres_u.data_ptr(),
-                        dec.centres_v.data_ptr(), n, m, x.data_ptr(), xp.data_ptr(), b, x.stride(0), y.data_ptr(),
-                        y.stride(0), _stream(stream))
+                        dec.centres_v.data_ptr(), n, m, x.data_ptr(), xp.data_ptr(), b, _ld(x), y.data_ptr(),
+                        _ld(y), _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_matmul_2bit")
     return y
@@ -466,16 +477,27 @@ def kd_matmul_2bit_f16_batch(mats, count, batch, stream) -> int:
     return lib.kd_matmul_2bit_f16_batch(mats, count, batch, stream)
 
 
+def kd_matmul_2bit_bf16(codes_u, codes_v, centres_u, centres_v, n, m, x, xp, batch, ldx, y, ldy, stream) -> int:
+    return lib.kd_matmul_2bit_bf16(codes_u, codes_v, centres_u, centres_v, n, m, x, xp, batch, ldx, y, ldy, stream)
+
+
+def kd_matmul_2bit_bf16_batch(mats, count, batch, stream) -> int:
+    return lib.kd_matmul_2bit_bf16_batch(mats, count, batch, stream)
+
+
 def matmul_2bit_f16(dec: "Decomposed", x, xp, out=None, stream=None):
-    """kd_matmul_2bit_f16: ``Y = X W_hat^T`` from the code planes on the tensor cores,
-    for fp16 ``x`` and ``xp`` (batch, n) CUDA tensors; returns (batch, m) fp32."""
+    """kd_matmul_2bit_f16 (or _bf16): ``Y = X W_hat^T`` from the code planes on the tensor
+    cores, for fp16 (or bf16) ``x`` and ``xp`` (batch, n) CUDA tensors; returns (batch, m) fp32."""
     return matmul_2bit_f16_batch([dec], [x], [xp], outs=None if out is None else [out], stream=stream)[0]
 
 
 def matmul_2bit_f16_batch(decs, xs, xps, outs=None, stream=None):
-    """kd_matmul_2bit_f16_batch: ``Y_i = X_i W_hat_i^T`` for several matrices, fp16
-    inputs (one batch size), one launch per 16 batch rows."""
+    """kd_matmul_2bit_f16_batch (or _bf16_batch, for bf16 inputs): ``Y_i = X_i W_hat_i^T``
+    for several matrices, 16-bit inputs of one type and batch size, one launch per 16 rows."""
     torch = _torch()
+    dt = xs[0].dtype
+    if dt not in (torch.float16, torch.bfloat16):
+        raise ValueError("x must be fp16 or bf16")
     if not 1 <= len(decs) <= KD_MAX_BATCH or len(xs) != len(decs) or len(xps) != len(decs):
         raise ValueError(f"1..{KD_MAX_BATCH} matrices with one x and one xp each")
     b = xs[0].shape[0]
@@ -483,20 +505,21 @@ def matmul_2bit_f16_batch(decs, xs, xps, outs=None, stream=None):
     res = []
     for i, (d, x, xp) in enumerate(zip(decs, xs, xps)):
         m, words = d.codes_u.shape
-        if x.dim() != 2 or x.shape[0] != b or x.dtype != torch.float16 or xp.shape != x.shape \
-                or xp.dtype != x.dtype or x.stride(1) != 1 or xp.stride(1) != 1 or x.stride(0) != xp.stride(0):
-            raise ValueError("x and xp must be fp16 (batch, n) tensors of one shape, unit inner stride")
+        if x.dim() != 2 or x.shape[0] != b or x.dtype != dt or xp.shape != x.shape \
+                or xp.dtype != x.dtype or x.stride(1) != 1 or xp.stride(1) != 1 or _ld(x) != _ld(xp):
+            raise ValueError("x and xp must be 16-bit (batch, n) tensors of one type and shape, unit inner stride")
         n = x.shape[1]
         if (n + 15) // 16 != words:
             raise ValueError("x does not match the code planes' vector length")
         y = outs[i] if outs is not None else torch.empty((b, m), dtype=torch.float32, device=x.device)
         arr[i] = KdFoldMatF16(d.codes_u.data_ptr(), d.codes_v.data_ptr(), d.centres_u.data_ptr(),
-                              d.centres_v.data_ptr(), x.data_ptr(), xp.data_ptr(), y.data_ptr(), n, m, x.stride(0),
-                              y.stride(0))
+                              d.centres_v.data_ptr(), x.data_ptr(), xp.data_ptr(), y.data_ptr(), n, m, _ld(x),
+                              _ld(y))
         res.append(y)
-    st = kd_matmul_2bit_f16_batch(ctypes.cast(arr, ctypes.c_void_p), len(decs), b, _stream(stream))
+    call = kd_matmul_2bit_bf16_batch if dt == torch.bfloat16 else kd_matmul_2bit_f16_batch
+    st = call(ctypes.cast(arr, ctypes.c_void_p), len(decs), b, _stream(stream))
     if st != KD_OK:
-        raise KashinError(st, "kd_matmul_2bit_f16_batch")
+        raise KashinError(st, "kd_matmul_2bit_bf16_batch" if dt == torch.bfloat16 else "kd_matmul_2bit_f16_batch")
     return res
 
 
@@ -516,14 +539,14 @@ def matmul_2bit_batch(decs, xs, xps, outs=None, stream=None):
     for i, (d, x, xp) in enumerate(zip(decs, xs, xps)):
         m, words = d.codes_u.shape
         if x.dim() != 2 or x.shape[0] != b or x.dtype != torch.float32 or xp.shape != x.shape \
-                or xp.dtype != x.dtype or x.stride(1) != 1 or xp.stride(1) != 1 or x.stride(0) != xp.stride(0):
+                or xp.dtype != x.dtype or x.stride(1) != 1 or xp.stride(1) != 1 or _ld(x) != _ld(xp):
             raise ValueError("x and xp must be fp32 (batch, n) tensors of one shape, unit inner stride")
         n = x.shape[1]
         if (n + 15) // 16 != words:
             raise ValueError("x does not match the code planes' vector length")
         y = outs[i] if outs is not None else torch.empty((b, m), dtype=torch.float32, device=x.device)
         arr[i] = KdFoldMat(d.codes_u.data_ptr(), d.codes_v.data_ptr(), d.centres_u.data_ptr(), d.centres_v.data_ptr(),
-                           x.data_ptr(), xp.data_ptr(), y.data_ptr(), n, m, x.stride(0), y.stride(0))
+                           x.data_ptr(), xp.data_ptr(), y.data_ptr(), n, m, _ld(x), _ld(y))
         res.append(y)
     st = kd_matmul_2bit_batch(ctypes.cast(arr, ctypes.c_void_p), len(decs), b, _stream(stream))
     if st != KD_OK:
@@ -611,7 +634,7 @@ def _host_descriptors(ws, sign_seeds, layout, outs):
         for t in (o.codes_u, o.codes_v, o.centres_u, o.centres_v, o.coeffs):
             if t is not None and t.is_cuda:
                 raise ValueError("outputs must be host tensors")
-        arr[i] = KdMatrixHost(w.data_ptr(), m, w.stride(0), int(sign_seeds[i]) & ((1 << 64) - 1),
+        arr[i] = KdMatrixHost(w.data_ptr(), m, _ld(w), int(sign_seeds[i]) & ((1 << 64) - 1),
                               _ptr(o.codes_u), _ptr(o.codes_v), _ptr(o.centres_u), _ptr(o.centres_v),
                               _ptr(o.coeffs))
     return arr, lay, n
@@ -681,7 +704,7 @@ def dequantise(codes, centres, n: int, dtype=None, layout: str = "rows", out=Non
     if out is None:
         out = torch.empty((m, n) if lay == KD_VEC_ROWS else (n, m), dtype=dtype, device=codes.device)
     st = kd_dequantise(codes.data_ptr(), centres.data_ptr(), n, m, _dtype_code(out.dtype), lay, out.data_ptr(),
-                       out.stride(0), _stream(stream))
+                       _ld(out), _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_dequantise")
     return out
@@ -705,7 +728,7 @@ def dequantise_batch(planes, n: int, dtype=None, layout: str = "rows", outs=None
             o = torch.empty((m, n) if lay == KD_VEC_ROWS else (n, m), dtype=dtype, device=codes.device)
         if o.dtype != dtype:
             raise ValueError("outputs must share one dtype")
-        arr[i] = KdPlane(codes.data_ptr(), centres.data_ptr(), o.data_ptr(), m, o.stride(0))
+        arr[i] = KdPlane(codes.data_ptr(), centres.data_ptr(), o.data_ptr(), m, _ld(o))
         res.append(o)
     st = kd_dequantise_batch(ctypes.cast(arr, ctypes.c_void_p), len(planes), n, _dtype_code(dtype), lay,
                              _stream(stream))
@@ -726,8 +749,8 @@ def rht(x, seed: int, inverse: bool = False, out=None, status=None, stream=None)
     y = out if out is not None else torch.empty((m, n), dtype=torch.float32, device=x.device)
     if y.dtype != torch.float32 or y.shape != x.shape or y.stride(1) != 1:
         raise ValueError("out must be an fp32 tensor of x's shape with unit inner stride")
-    st = kd_rht(x.data_ptr(), _dtype_code(x.dtype), n, m, x.stride(0), seed, 1 if inverse else 0, y.data_ptr(),
-                y.stride(0), status.data_ptr() if status is not None else None, _stream(stream))
+    st = kd_rht(x.data_ptr(), _dtype_code(x.dtype), n, m, _ld(x), seed, 1 if inverse else 0, y.data_ptr(),
+                _ld(y), status.data_ptr() if status is not None else None, _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_rht")
     return y
@@ -746,7 +769,7 @@ def reconstruct(dec: Decomposed, n: int, sign_seed: int, dtype=None, layout: str
     ws = workspace if workspace is not None else Workspace(n, dev)
     st = kd_reconstruct(dec.codes_u.data_ptr(), dec.codes_v.data_ptr(), dec.centres_u.data_ptr(),
                         dec.centres_v.data_ptr(), n, m, sign_seed, _dtype_code(out.dtype), lay, out.data_ptr(),
-                        out.stride(0), ws.ptr, ws.nbytes, _stream(stream))
+                        _ld(out), ws.ptr, ws.nbytes, _stream(stream))
     if st != KD_OK:
         raise KashinError(st, "kd_reconstruct")
     return out
@@ -771,7 +794,7 @@ def reconstruct_batch(decs, n: int, sign_seeds, dtype=None, layout: str = "rows"
         if o.dtype != dtype:
             raise ValueError("outputs must share one dtype")
         arr[i] = KdRecMat(d.codes_u.data_ptr(), d.codes_v.data_ptr(), d.centres_u.data_ptr(), d.centres_v.data_ptr(),
-                          int(sign_seeds[i]) & ((1 << 64) - 1), o.data_ptr(), m, o.stride(0))
+                          int(sign_seeds[i]) & ((1 << 64) - 1), o.data_ptr(), m, _ld(o))
         res.append(o)
     ws = workspace if workspace is not None else Workspace(n, dev, count=len(decs))
     st = kd_reconstruct_batch(ctypes.cast(arr, ctypes.c_void_p), len(decs), n, _dtype_code(dtype), lay, ws.ptr,

@@ -341,6 +341,11 @@ def test_matmul_2bit_f16_validation(kd):
     assert kd.kd_matmul_2bit_f16_batch(arr, 2, 1, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_matmul_2bit_f16_batch(arr, 2, 0, null) == kd.KD_ERR_INVALID_ARG       # checked even when empty
     assert kd.kd_matmul_2bit_f16_batch(arr, 1, 0, null) == kd.KD_OK
+    fb = kd.kd_matmul_2bit_bf16
+    assert fb(16, 16, 16, 16, 0, 4, 16, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG      # n = 0
+    assert fb(16, 16, 16, 16, 256, 4, 17, 16, 1, 256, 16, 4, null) == kd.KD_ERR_INVALID_ARG    # x odd address
+    assert fb(null, null, null, null, 256, 4, null, null, 0, 256, null, 4, null) == kd.KD_OK   # batch == 0
+    assert kd.kd_matmul_2bit_bf16_batch(arr, 2, 1, null) == kd.KD_ERR_INVALID_ARG
 
 
 def test_prepared_p_validation(kd):
@@ -382,3 +387,14 @@ def test_batched_product_and_transform_validation(kd):
     assert kd.kd_apply_p_batch(parr, 1, 4094, 16, 1 << 20, null) == kd.KD_ERR_UNSUPPORTED_N
     assert kd.kd_apply_p_batch(parr, 2, 256, 16, 1 << 20, null) == kd.KD_ERR_INVALID_ARG
     assert kd.kd_apply_p_batch(parr, 1, 256, null, 1 << 20, null) == kd.KD_ERR_WORKSPACE
+
+
+def test_binding_leading_dimension_of_one_row(kd):
+    """A one-row tensor may carry any row stride (numpy and torch treat it as contiguous
+    either way); the binding then passes the row length as the leading dimension, which
+    every entry point accepts.  Several rows keep their own stride."""
+    import torch
+    one = torch.zeros(10).as_strided((1, 10), (1, 1))
+    assert kd._ld(one) == 10
+    assert kd._ld(torch.zeros((3, 12))[:, :10]) == 12
+

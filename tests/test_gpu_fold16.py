@@ -1,4 +1,4 @@
-"""kd_matmul_2bit_f16: the folded layer product (App. C) for fp16 activations on the
+"""kd_matmul_2bit_f16 and _bf16: the folded layer product (App. C) for 16-bit activations on the
 tensor cores, against the fp64 oracle.
 
 Both sides use the device decomposition's codes and centres (which codes a
@@ -57,16 +57,22 @@ def _h(a):
     return np.asarray(a, dtype=np.float64).astype(np.float16).astype(np.float64)
 
 
-def _exact(kd, w, seed, batch, iters=8, gen_seed=0):
+def _hb(a):
+    """bf16 rounding (nearest, ties to even, by torch on the host), back in fp64."""
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float64)).to(torch.bfloat16).double().numpy()
+
+
+def _exact(kd, w, seed, batch, iters=8, gen_seed=0, bf16=False):
     m, n = w.shape
+    dt, rnd = (torch.bfloat16, _hb) if bf16 else (torch.float16, _h)
     dec = kd.decompose(w, iters, seed)
     g = torch.Generator().manual_seed(gen_seed)
-    x16 = torch.randn((batch, n), generator=g).half()
-    xp16 = torch.from_numpy(np.ascontiguousarray(_h(_pop(n, seed)(x16.double().numpy().T).T))).half()
+    x16 = torch.randn((batch, n), generator=g).to(dt)
+    xp16 = torch.from_numpy(np.ascontiguousarray(rnd(_pop(n, seed)(x16.double().numpy().T).T))).to(dt)
     y = kd.matmul_2bit_f16(dec, x16.cuda(), xp16.cuda())
     torch.cuda.synchronize()
     cu, cv = _planes(kd, dec, n)
-    y_ora = x16.double().numpy() @ _h(cu) + xp16.double().numpy() @ _h(cv)
+    y_ora = x16.double().numpy() @ rnd(cu) + xp16.double().numpy() @ rnd(cv)
     err = np.abs(y.double().cpu().numpy() - y_ora).max(axis=1)
     scale = np.abs(y_ora).max(axis=1)
     assert (err <= TOL * scale).all(), (err / scale).max()
@@ -164,3 +170,37 @@ def test_f16_strided_rows(kd):
         torch.cuda.synchronize()
         assert torch.equal(ys[:, :m], ref)
         assert torch.isnan(ys[:, m:]).all()
+
+
+@pytest.mark.parametrize("name,batch", [("L0.q", 1), ("L0.down", 9), ("L0.gate", 16)])
+def test_bf16_exact_inputs(kd, name, batch):
+    """kd_matmul_2bit_bf16: the same exact-input parity with bf16 activations and centres
+    rounded to bf16 on both sides."""
+    spec = {s.name: s for s in synth.config3()}[name]
+    w = synth.generate(spec, device="cuda")
+    _exact(kd, w, spec.sign_seed, batch, iters=16, gen_seed=batch, bf16=True)
+
+
+def test_bf16_ragged_and_end_to_end(kd):
+    """bf16 on a ragged case (partial tiles, a partial code word, 17 rows) and end to end
+    from fp32 X against the full-precision product, within the bf16 rounding bound
+    1.01 * 2^-8 * sum_i (|x_i u_i| + |xp_i v_i|) plus 1e-5 of max |Y|."""
+    g = torch.Generator(device="cuda").manual_seed(5)
+    w = (torch.randn((19, 1000), generator=g, device="cuda") * 0.02).half()
+    _exact(kd, w, 7, 17, gen_seed=3, bf16=True)
+    spec = {s.name: s for s in synth.config3()}["L0.q"]
+    w = synth.generate(spec, device="cuda")
+    n = spec.N
+    dec = kd.decompose(w, 16, spec.sign_seed)
+    x = torch.randn((3, n), generator=g, device="cuda")
+    xp = kd.apply_p(x, spec.sign_seed)
+    y = kd.matmul_2bit_f16(dec, x.bfloat16(), xp.bfloat16())
+    torch.cuda.synchronize()
+    cu, cv = _planes(kd, dec, n)
+    x64 = x.double().cpu().numpy()
+    xp64 = _pop(n, spec.sign_seed)(x64.T).T
+    y_ora = x64 @ cu + xp64 @ cv
+    bound = 1.01 * 2.0 ** -8 * (np.abs(x64) @ np.abs(cu) + np.abs(xp64) @ np.abs(cv))
+    bound += TOL * np.abs(y_ora).max(axis=1, keepdims=True)
+    assert (np.abs(y.double().cpu().numpy() - y_ora) <= bound).all()
+
