@@ -104,8 +104,8 @@ __device__ __forceinline__ float2 cscale(float2 a, float s) {
 __device__ __forceinline__ float2 mul_mi(float2 a) { return make_float2(a.y, -a.x); }
 // +i * a   (exact)
 __device__ __forceinline__ float2 mul_pi(float2 a) { return make_float2(-a.y, a.x); }
-// a + i b and a - i b as two scalar adds: the swapped operand would need register
-// moves in packed form.
+// a + i b and a - i b as two scalar adds (the packed forms below, one instruction each,
+// are used by the plans with packed constant roots and by Rader's form).
 __device__ __forceinline__ float2 add_ib(float2 a, float2 b) {
   return make_float2(__fsub_rn(a.x, b.y), __fadd_rn(a.y, b.x));
 }
@@ -115,6 +115,14 @@ __device__ __forceinline__ float2 sub_ib(float2 a, float2 b) {
 // swapped pair: packed FP32x2 instructions read either half of a register pair for
 // either lane, so (a.y, a.x) as an operand costs no instruction (measured on sm_103a)
 __device__ __forceinline__ float2 swp(float2 a) { return make_float2(a.y, a.x); }
+// a + i b and a - i b as one packed FMA on the swapped pair (b times +-1 is exact, so
+// each lane rounds once, exactly as the scalar forms)
+__device__ __forceinline__ float2 add_ib_pk(float2 a, float2 b) {
+  return __ffma2_rn(swp(b), make_float2(-1.f, 1.f), a);
+}
+__device__ __forceinline__ float2 sub_ib_pk(float2 a, float2 b) {
+  return __ffma2_rn(swp(b), make_float2(1.f, -1.f), a);
+}
 
 // Multiply by the compile-time root W_R^E = exp(DIR * 2 pi i E / R), DIR = -1 forward.
 // Quarter turns are exact; eighth turns use one constant; others a full product.
@@ -213,7 +221,10 @@ struct Dft<4, DIR, PK> {
     // forward: X1 = d02 - i d13, X3 = d02 + i d13 ; inverse: signs swapped
     v[0] = cadd(s02, s13);
     v[2] = csub(s02, s13);
-    if constexpr (DIR < 0) {
+    if constexpr (PK) {
+      v[1] = DIR < 0 ? sub_ib_pk(d02, d13) : add_ib_pk(d02, d13);
+      v[3] = DIR < 0 ? add_ib_pk(d02, d13) : sub_ib_pk(d02, d13);
+    } else if constexpr (DIR < 0) {
       v[1] = sub_ib(d02, d13);
       v[3] = add_ib(d02, d13);
     } else {
@@ -225,7 +236,7 @@ struct Dft<4, DIR, PK> {
 
 // Odd prime R: symmetric direct form.  a_n = x_n + x_{R-n}, b_n = x_n - x_{R-n};
 // X_k = x_0 + sum a_n cos(2 pi n k / R) -+ i sum b_n sin(2 pi n k / R).
-template <int R, int DIR>
+template <int R, int DIR, bool PK = false>
 struct DftPrime {
   template <class Arr>
   __device__ __forceinline__ static void run(Arr& v) {
@@ -252,7 +263,10 @@ struct DftPrime {
         bk = __ffma2_rn(b[NN], make_float2(s, s), bk);
       });
       // forward: X_k = ak - i bk, X_{R-k} = ak + i bk ; inverse: the reverse
-      if constexpr (DIR < 0) {
+      if constexpr (PK) {
+        v[K] = DIR < 0 ? sub_ib_pk(ak, bk) : add_ib_pk(ak, bk);
+        v[R - K] = DIR < 0 ? add_ib_pk(ak, bk) : sub_ib_pk(ak, bk);
+      } else if constexpr (DIR < 0) {
         v[K] = sub_ib(ak, bk);
         v[R - K] = add_ib(ak, bk);
       } else {
@@ -330,7 +344,9 @@ KD_HD constexpr bool kd_is_big_prime() {
 // prime-factor (Good-Thomas) A x B DFT without twiddles.
 //
 // Per point of a 43-point DFT this is about 35 FMA-pipe operations against 46 for the
-// symmetric direct form, with independent butterflies instead of 21-term chains.
+// symmetric direct form, with independent butterflies instead of 21-term chains.  The
+// spectrum products and the final a +- i b run as packed FP32x2 instructions, which keeps
+// the code (and the instruction-cache footprint of the kernel) small.
 // ---------------------------------------------------------------------------
 KD_HD constexpr long long kd_powmod(long long b, long long e, long long m) {
   long long r = 1;
@@ -395,24 +411,25 @@ __device__ __forceinline__ void dft_pfa(Arr& y) {
     constexpr int N2 = decltype(n2c)::value;
     float2 s[A];
     static_for<0, A>([&](auto n1c) { s[decltype(n1c)::value] = y[(B * decltype(n1c)::value + A * N2) % N]; });
-    Dft<A, SGN>::run(s);
+    Dft<A, SGN, true>::run(s);
     static_for<0, A>([&](auto k1c) { t[decltype(k1c)::value * B + N2] = s[decltype(k1c)::value]; });
   });
   static_for<0, A>([&](auto k1c) {
     constexpr int K1 = decltype(k1c)::value;
     float2 s[B];
     static_for<0, B>([&](auto n2c) { s[decltype(n2c)::value] = t[K1 * B + decltype(n2c)::value]; });
-    Dft<B, SGN>::run(s);
+    Dft<B, SGN, true>::run(s);
     static_for<0, B>([&](auto k2c) { y[(ka * K1 + kb * decltype(k2c)::value) % N] = s[decltype(k2c)::value]; });
   });
 }
 
-// a * (c + i s) with compile-time c, s (four scalar operations)
+// a * (c + i s) with compile-time c, s: two packed operations on the swapped pair (the
+// constants carry the sign, so no operand needs negating)
 template <int R, int KIND, int K>
 __device__ __forceinline__ float2 mul_rader_spectrum(float2 a) {
   constexpr float c = (float)kd_rader_spectrum<R, KIND, false>(K);
   constexpr float s = (float)kd_rader_spectrum<R, KIND, true>(K);
-  return make_float2(__fmaf_rn(a.x, c, __fmul_rn(-a.y, s)), __fmaf_rn(a.x, s, __fmul_rn(a.y, c)));
+  return __ffma2_rn(swp(a), make_float2(-s, s), __fmul2_rn(a, make_float2(c, c)));
 }
 
 // Streaming form, the same interface as dft_prime_stream: every input is read once
@@ -456,11 +473,11 @@ __device__ __forceinline__ void dft_prime_rader(Load&& load, Store&& store) {
     constexpr int k = (int)kd_powmod(g, M, R);
     // X(k_m) = P_m + s i Q'_m with s = DIR (-1)^m
     if constexpr ((DIR < 0) != ((M & 1) != 0)) {
-      store(ic<k>{}, sub_ib(u[M], w[M]));
-      store(ic<R - k>{}, add_ib(u[M], w[M]));
+      store(ic<k>{}, sub_ib_pk(u[M], w[M]));
+      store(ic<R - k>{}, add_ib_pk(u[M], w[M]));
     } else {
-      store(ic<k>{}, add_ib(u[M], w[M]));
-      store(ic<R - k>{}, sub_ib(u[M], w[M]));
+      store(ic<k>{}, add_ib_pk(u[M], w[M]));
+      store(ic<R - k>{}, sub_ib_pk(u[M], w[M]));
     }
   });
 }
@@ -514,7 +531,7 @@ struct Dft {
   template <class A>
   __device__ __forceinline__ static void run(A& v) {
     if constexpr (SmallestFactor<R>::value == R) {
-      DftPrime<R, DIR>::run(v);
+      DftPrime<R, DIR, PK>::run(v);
     } else {
       DftComposite<R, DIR, PK>::run(v);
     }
