@@ -32,8 +32,9 @@
  *              work on the stream and return.
  *  Errors      argument / size / plan problems are returned synchronously and
  *              nothing is enqueued; a failed launch returns KD_ERR_CUDA; a
- *              non-finite input value is detected on the device and reported
- *              by kd_read_status().  No call traps or aborts.
+ *              non-finite input value, or a bounded wait that expired (the CTA
+ *              then leaves its remaining vectors unwritten), is detected on the
+ *              device and reported by kd_read_status().  No call traps or aborts.
  *  Supported n: 1 <= n <= 16384 whose prime factors all lie in
  *              {2, 3, 5, 7, 11, 13, 43} (kd_supported()).  Sixteen lengths have a
  *              compiled, tuned plan (kd_tuned()): 16, 32, 64, 128, 256, 512, 768,
@@ -59,7 +60,8 @@ typedef enum {
   KD_ERR_UNSUPPORTED_N = 2, /* vector length outside the supported set (see "Supported n") */
   KD_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed */
   KD_ERR_NONFINITE = 4,     /* a decomposed vector held NaN or Inf (device-detected) */
-  KD_ERR_WORKSPACE = 5      /* workspace pointer null, not 16-byte aligned, or too small */
+  KD_ERR_WORKSPACE = 5,     /* workspace pointer null, not 16-byte aligned, or too small */
+  KD_ERR_TIMEOUT = 6        /* a bounded wait inside a kernel expired (device-detected) */
 } kd_status;
 
 typedef enum { KD_F32 = 0, KD_F16 = 1, KD_BF16 = 2 } kd_dtype;
@@ -157,9 +159,9 @@ kd_status kd_decompose_static(const void* w, kd_dtype dtype, kd_layout layout, i
                               void* stream);
 
 /* kd_read_status for kd_decompose_static: synchronises `stream`, then returns
- * KD_ERR_NONFINITE if a vector of the last kd_decompose_static call on the current
- * device held a NaN or Inf, KD_OK otherwise (also when no static call ran yet), and
- * KD_ERR_CUDA if a CUDA call fails.  Allocates nothing.  The word is shared like the
+ * KD_ERR_TIMEOUT or KD_ERR_NONFINITE as kd_read_status does for the last
+ * kd_decompose_static call on the current device, KD_OK otherwise (also when no
+ * static call ran yet), and KD_ERR_CUDA if a CUDA call fails.  Allocates nothing.  The word is shared like the
  * rest of the array: a static call enqueued after the one of interest clears it. */
 kd_status kd_read_status_static(void* stream);
 
@@ -315,9 +317,11 @@ typedef struct kd_recmat {
 kd_status kd_reconstruct_batch(const kd_recmat* mats, int count, int64_t n, kd_dtype out_dtype, kd_layout layout,
                                void* workspace, size_t ws_bytes, void* stream);
 
-/* Synchronises `stream` and returns KD_ERR_NONFINITE if any vector decomposed
- * by the last kd_decompose on this workspace held a NaN or Inf, KD_OK otherwise
- * (KD_ERR_CUDA if the synchronisation fails). */
+/* Synchronises `stream` and reads the status word of the last kd_decompose (or
+ * kd_decompose_batch) on this workspace: KD_ERR_TIMEOUT if a staged-input copy did
+ * not complete within the kernel's bounded wait (about a second; that CTA's
+ * remaining vectors are not written), else KD_ERR_NONFINITE if any vector held a
+ * NaN or Inf, KD_OK otherwise (KD_ERR_CUDA if the synchronisation fails). */
 kd_status kd_read_status(const void* workspace, void* stream);
 
 /* Dequantise one 2-bit factor plane (App. C, inference): out entry i of vector j =

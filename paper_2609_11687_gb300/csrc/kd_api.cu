@@ -196,6 +196,7 @@ const char* kd_status_string(kd_status s) {
     case KD_ERR_CUDA: return "KD_ERR_CUDA";
     case KD_ERR_NONFINITE: return "KD_ERR_NONFINITE";
     case KD_ERR_WORKSPACE: return "KD_ERR_WORKSPACE";
+    case KD_ERR_TIMEOUT: return "KD_ERR_TIMEOUT";
     default: return "KD_ERR_UNKNOWN";
   }
 }
@@ -600,7 +601,9 @@ kd_status kd_read_status(const void* workspace, void* stream) {
   uint32_t word = 0;
   if (cudaMemcpyAsync(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost, s) != cudaSuccess) return KD_ERR_CUDA;
   if (cudaStreamSynchronize(s) != cudaSuccess) return KD_ERR_CUDA;
-  return word ? KD_ERR_NONFINITE : KD_OK;
+  // bit 1: a staged-input wait expired; bit 0: a non-finite input
+  if (word & 2u) return KD_ERR_TIMEOUT;
+  return (word & 1u) ? KD_ERR_NONFINITE : KD_OK;
 }
 
 }  // extern "C"

@@ -25,7 +25,7 @@ import numpy as np
 HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libkashin.so")
 
-KD_OK, KD_ERR_INVALID_ARG, KD_ERR_UNSUPPORTED_N, KD_ERR_CUDA, KD_ERR_NONFINITE, KD_ERR_WORKSPACE = range(6)
+KD_OK, KD_ERR_INVALID_ARG, KD_ERR_UNSUPPORTED_N, KD_ERR_CUDA, KD_ERR_NONFINITE, KD_ERR_WORKSPACE, KD_ERR_TIMEOUT = range(7)
 KD_F32, KD_F16, KD_BF16 = 0, 1, 2
 KD_VEC_ROWS, KD_VEC_COLUMNS = 0, 1
 

@@ -47,6 +47,7 @@ def test_version_and_status_strings(kd):
     assert "libkashin" in kd.version()
     assert kd.status_string(kd.KD_OK) == "KD_OK"
     assert kd.status_string(kd.KD_ERR_NONFINITE) == "KD_ERR_NONFINITE"
+    assert kd.status_string(kd.KD_ERR_TIMEOUT) == "KD_ERR_TIMEOUT"
     assert kd.status_string(99) == "KD_ERR_UNKNOWN"
 
 

@@ -190,6 +190,22 @@ def test_nonfinite_input_sets_status(kd, torch_mod):
     assert kd.read_status(ws) == kd.KD_OK
 
 
+def test_read_status_decodes_the_word(kd, torch_mod):
+    """kd_read_status decodes the workspace's status word: bit 1 (a staged-input wait
+    that expired) reads as KD_ERR_TIMEOUT, also together with bit 0; bit 0 alone as
+    KD_ERR_NONFINITE; and the next decomposition clears the word.  The bits are written
+    into the word directly: no wait is made to expire."""
+    torch = torch_mod
+    ws = kd.Workspace(256)
+    word = ws.buf[:4].view(torch.int32)
+    for bits, want in ((2, kd.KD_ERR_TIMEOUT), (3, kd.KD_ERR_TIMEOUT), (1, kd.KD_ERR_NONFINITE), (0, kd.KD_OK)):
+        word.fill_(bits)
+        assert kd.read_status(ws) == want
+    word.fill_(2)
+    kd.decompose(_rand(torch, (4, 256), seed=2).cuda(), 4, 0, workspace=ws)
+    assert kd.read_status(ws) == kd.KD_OK
+
+
 def test_deterministic(kd, torch_mod):
     torch = torch_mod
     w = _rand(torch, (64, 4096), seed=31, dtype=torch.float16).cuda()
