@@ -4,8 +4,9 @@
 //     y[r][j] = sum_i h(cu_j[code_u(j, i)]) x[r][i] + sum_i h(cv_j[code_v(j, i)]) xp[r][i]
 //
 // with x, xp in the 16-bit type (xp = X P from kd_apply_p, rounded by the caller), h()
-// the rounding of a centre to that type, fp32 accumulation.  Neither plane is expanded in memory: each
-// code becomes its fp16 centre in registers and feeds an mma.sync B fragment directly.
+// the rounding of a centre to that type, fp32 accumulation.  Neither plane is expanded
+// in memory: each code becomes its 16-bit centre in registers and feeds an mma.sync B
+// fragment directly.
 //
 // Mapping.  mma.m16n8k16 with M = the batch rows (up to 16 per launch), N = 8 output
 // channels, K = 16 inputs.  A work item is a tile of 32 channels (four n-tiles) of one
@@ -24,9 +25,9 @@
 // its B fragments are code word t of the group (inputs 16 t .. 16 t + 15) of its
 // channel: byte j of that word holds the four codes of k-step j.
 //
-// Decoding.  The four fp16 centres of a channel are kept as two words, L (their low
+// Decoding.  The four 16-bit centres of a channel are kept as two words, L (their low
 // bytes) and H (their high bytes).  For two codes q0, q1 one byte permute with the
-// selector nibbles (q0, q0 + 4, q1, q1 + 4) yields the fp16 pair (c[q0], c[q1]); the
+// selector nibbles (q0, q0 + 4, q1, q1 + 4) yields the pair (c[q0], c[q1]); the
 // selectors of two k-steps are formed together from one shifted code word.
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
