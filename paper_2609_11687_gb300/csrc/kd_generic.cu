@@ -96,16 +96,16 @@ __device__ __forceinline__ void gen_pass_r(float2* buf, const float2* __restrict
     const int sp = g - blk * S;
     const int base = blk * Bk + sp;
     if constexpr (kd_is_big_prime<R>()) {
-      // streaming form: every load of the group precedes its first store
+      // streaming form (Rader's for 43, direct otherwise): every load precedes the first store
       if constexpr (DIR < 0) {
-        dft_prime_stream<R, -1>([&](auto jc) { return buf[pad(base + decltype(jc)::value * S)]; },
+        dft_prime_pass<R, -1>([&](auto jc) { return buf[pad(base + decltype(jc)::value * S)]; },
                                 [&](auto kc, float2 x) {
                                   constexpr int K = decltype(kc)::value;
                                   if (K > 0 && !last) x = cmul(x, __ldg(&tw[K * S + sp]));
                                   buf[pad(base + K * S)] = x;
                                 });
       } else {
-        dft_prime_stream<R, +1>(
+        dft_prime_pass<R, +1>(
             [&](auto jc) {
               constexpr int J = decltype(jc)::value;
               float2 x = buf[pad(base + J * S)];
