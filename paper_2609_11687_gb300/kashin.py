@@ -10,7 +10,12 @@ Two layers:
 
 * ``kd_*`` functions mirror the C entry points one to one (raw device pointers
   as Python ints, a status code back);
-* ``decompose`` / ``apply_p`` / ``reconstruct`` take and return torch tensors.
+* tensor-level wrappers take and return torch tensors: ``decompose`` (and
+  ``decompose_batch``, ``decompose_batch_host``), ``apply_p`` (``apply_p_batch``,
+  ``prepare_p`` + ``apply_p_prepared``), ``reconstruct`` (``reconstruct_batch``),
+  ``dequantise`` (``dequantise_batch``), ``rht``, and the products from the 2-bit
+  planes ``matmul_2bit`` (fp32) and ``matmul_2bit_f16`` (fp16 or bf16 activations,
+  tensor cores), each with a ``_batch`` form.
 """
 
 from __future__ import annotations
