@@ -65,11 +65,11 @@ def test_matmul_2bit_7b_shapes(kd, name, batch):
     _run(kd, w, spec.sign_seed, batch, gen_seed=batch)
 
 
-@pytest.mark.parametrize("n,m,batch", [(768, 37, 6), (1000, 19, 5), (256, 1, 2), (16, 9, 1)])
+@pytest.mark.parametrize("n,m,batch", [(768, 37, 6), (1000, 19, 5), (256, 1, 2), (16, 9, 1), (16384, 21, 3)])
 def test_matmul_2bit_ragged(kd, n, m, batch):
     """Channel counts that leave a partial tile, a length with a partial last code word
-    (run-time-length path), a single channel, the shortest length; batch chunks 4+2,
-    4+1, 2, 1."""
+    (run-time-length path), a single channel, the shortest and the longest lengths; batch
+    chunks 2+2+2, 2+2+1, 2, 1 and 2+1."""
     g = torch.Generator(device="cuda").manual_seed(n + m)
     w = (torch.randn((m, n), generator=g, device="cuda") * 0.02).half()
     _run(kd, w, 7, batch)

@@ -8,7 +8,10 @@ is checked here.
 * Exact inputs: the test draws X in fp16, the oracle forms X P in fp64 and rounds it to
   fp16 (numpy, nearest-even), and both sides take those same fp16 rows.  The oracle
   rounds the centres to fp16 the same way, so the only difference left is the fp32
-  summation: tolerance 1e-5 of max |Y| per batch row.
+  summation: tolerance 1e-5 of max |Y| per batch row for n <= 4096.  For terms of random
+  sign that summation error grows like sqrt(n) relative to |Y| (the partial sums walk
+  like sqrt(k)), so longer vectors get 1e-5 sqrt(n / 4096): 1.6e-5 at n = 11008, 2e-5 at
+  16384, where the tensor cores' sums over 256 k-steps per warp measured 1.16e-5.
 * End to end: fp32 X, X P from kd_apply_p, both rounded to fp16 by torch, against the
   full-precision fp64 product.  Rounding an input and a centre to fp16 changes each term
   x_i c_i by at most (2^-10 + 2^-22) |x_i c_i|, so the bound is 1.01 * 2^-10 * sum_i
@@ -75,7 +78,8 @@ def _exact(kd, w, seed, batch, iters=8, gen_seed=0, bf16=False):
     y_ora = x16.double().numpy() @ rnd(cu) + xp16.double().numpy() @ rnd(cv)
     err = np.abs(y.double().cpu().numpy() - y_ora).max(axis=1)
     scale = np.abs(y_ora).max(axis=1)
-    assert (err <= TOL * scale).all(), (err / scale).max()
+    tol = TOL * max(1.0, (n / 4096) ** 0.5)
+    assert (err <= tol * scale).all(), (err / scale).max()
     return dec, y
 
 
@@ -203,4 +207,13 @@ def test_bf16_ragged_and_end_to_end(kd):
     bound = 1.01 * 2.0 ** -8 * (np.abs(x64) @ np.abs(cu) + np.abs(xp64) @ np.abs(cv))
     bound += TOL * np.abs(y_ora).max(axis=1, keepdims=True)
     assert (np.abs(y.double().cpu().numpy() - y_ora) <= bound).all()
+
+
+@pytest.mark.parametrize("bf16", [False, True])
+def test_f16_longest_length(kd, bf16):
+    """The longest supported vector length (n = 16384, 1,024 code words per channel) with a
+    full 16-row batch and a partial 32-channel tile."""
+    g = torch.Generator(device="cuda").manual_seed(16384)
+    w = (torch.randn((45, 16384), generator=g, device="cuda") * 0.02).half()
+    _exact(kd, w, 21, 16, gen_seed=7, bf16=bf16)
 
