@@ -399,3 +399,27 @@ def test_binding_leading_dimension_of_one_row(kd):
     assert kd._ld(one) == 10
     assert kd._ld(torch.zeros((3, 12))[:, :10]) == 12
 
+
+def test_wrappers_refuse_bad_tensors_before_any_cuda_call(kd):
+    """The tensor-level wrappers of the 16-bit product and of the prepared P check dtypes,
+    shapes and counts on the host and raise ValueError before touching the device."""
+    import pytest
+    import torch
+
+    class Planes:  # only the code-plane shape is read before the checks fail
+        codes_u = torch.zeros((4, 16), dtype=torch.int32)
+
+    d = [Planes()]
+    f32, f16, bf16 = (torch.zeros((1, 256), dtype=t) for t in (torch.float32, torch.float16, torch.bfloat16))
+    with pytest.raises(ValueError):
+        kd.matmul_2bit_f16_batch(d, [f32], [f32])               # fp32 activations
+    with pytest.raises(ValueError):
+        kd.matmul_2bit_f16_batch(d, [f16], [bf16])              # mixed 16-bit types
+    with pytest.raises(ValueError):
+        kd.matmul_2bit_f16_batch(d, [torch.zeros((1, 240), dtype=torch.float16)] * 1,
+                                 [torch.zeros((1, 240), dtype=torch.float16)])  # n does not match the planes
+    with pytest.raises(ValueError):
+        kd.prepare_p(256, list(range(33)))                      # more than 32 sign sets
+    with pytest.raises(ValueError):
+        kd.apply_p_prepared([f16], None)                        # P takes fp32 rows
+
